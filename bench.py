@@ -1,0 +1,527 @@
+#!/usr/bin/env python3
+"""Benchmark of the canary-trap verifier hot path on GB300.
+
+One step = one pass of the verifier over one synthetic pipeline already
+resident in HBM: the drift reduction of every (stage, canary) segment
+(relative-L2 of Eq. 4, max-abs, cosine mismatch), the scrambled-label
+control labels (Sec. 4.5) and the Mann-Whitney AUROC (Eq. 5-6) of the true
+and the control labels.  The pipeline itself (fp32 references and fp16 live
+activations) is materialised on the device by the generator before the timed
+region; its own throughput is reported under "generate".
+
+Output: one JSON line (rank 0).  `value` = canary activation elements scored
+per second over all ranks.  `roofline` is the drift kernel's algorithmic HBM
+bytes (6 per element: 2 fp16 + 4 fp32, each read once) per launch over its
+CUDA-event duration, against the measured copy bandwidth.  `e2e` repeats the
+step with the inputs in pinned host memory, copied in every step, and the
+scores and A-hat copied back.  `cpu_baseline` times the fp64 CPU oracle on a
+bounded sample of the same workload.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 70b|7b|paper_shape|tiny]
+  python bench.py --impl reference ...   (times the CPU oracle as the reference arm)
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import seeded_inputs as SI  # noqa: E402
+
+WORKLOAD_NAMES = {
+    "70b": "70B-like pipeline: 16 stages x hidden 8192, 256 canaries x 128 tokens, fp16 live / fp32 "
+           "references, benign noise 2e-3 (Eq. 2), stage 8 (1-based) flips the sign of 1% of channels, seed 2",
+    "7b": "7B-like pipeline: 8 stages x hidden 4096, 64 canaries x 128 tokens, 4 outlier channels x20, "
+          "benign noise 1e-3 (Eq. 2), Gaussian tamper 1e-2 on stage 4 (1-based), seed 1",
+    "paper_shape": "paper-shape pipeline: 12 stages x hidden 768, 100 canaries x 48 tokens, sigma_hw 2e-3, "
+                   "Gaussian tamper 0.05 on stage 6 (1-based), seed 5",
+    "tiny": "tiny pipeline: 4 stages x hidden 256, 16 canaries x 32 tokens, seed 0",
+}
+WORKLOADS = {"70b": SI.SEVENTY_B, "7b": SI.SEVEN_B, "paper_shape": SI.PAPER_SHAPE, "tiny": SI.TINY}
+METRIC = "canary activation elements scored/sec (HBM GB/s vs peak); AUROC configs/sec"
+BYTES_PER_ELEMENT = 6          # 2 B fp16 live + 4 B fp32 reference, each read once
+L2_BYTES = 129 * 2**20
+
+
+def parse_args(argv=None):
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=int(os.environ.get("WORLD_SIZE", "1")))
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--workload", default="70b", choices=sorted(WORKLOADS))
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=10.0,
+                   help="target duration of the timed CPU-oracle sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args(argv)
+
+
+# ----------------------------------------------------------------------------- ranks
+
+class Ranks:
+    """One process per GPU (torchrun); timing = max over ranks."""
+
+    def __init__(self):
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.pg = None
+
+    def init(self, backend):
+        if self.world > 1:
+            import torch.distributed as dist
+            os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+            dist.init_process_group(backend=backend)
+            self.pg = dist
+
+    def barrier(self):
+        if self.pg:
+            self.pg.barrier()
+
+    def max(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        dev = "cuda" if self.pg.get_backend() == "nccl" else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum(self, x: float) -> float:
+        if not self.pg:
+            return x
+        import torch
+        dev = "cuda" if self.pg.get_backend() == "nccl" else "cpu"
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        self.pg.all_reduce(t, op=self.pg.ReduceOp.SUM)
+        return float(t.item())
+
+    def close(self):
+        if self.pg:
+            self.pg.destroy_process_group()
+
+
+def rank_config(cfg: dict, rank: int) -> dict:
+    """Weak scaling: rank r scores its own independent pipeline (config id + r)."""
+    return SI.shrink(cfg, config_id=cfg["config_id"] + rank)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- peaks
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def recorded_traffic(kernel_src: str, profile_name: str):
+    """dram bytes per launch recorded by the committed ncu summary, when the
+    kernel source still has the hash recorded there; else None."""
+    path = os.path.join(ROOT, "profiles", profile_name)
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m_t = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    m_h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
+    if not (m_t and m_h):
+        return None
+    src = open(os.path.join(ROOT, "paper_2607_19490_gb300", "csrc", kernel_src), "rb").read()
+    if hashlib.sha256(src).hexdigest() != m_h.group(1):
+        return None
+    return float(m_t.group(1))
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+
+def oracle_prepare(cfg, n_threads):
+    """A bounded sample of the workload for the fp64 CPU oracle: every stage x
+    the first few canaries (about 256 Mi elements at most), generated by the
+    oracle's own generator (untimed)."""
+    from oracle import oracle as O
+    O.build()
+    S, L = cfg["n_shards"], cfg["tokens"] * cfg["hidden"]
+    n_can = max(1, min(cfg["n_canaries"], (256 * 2**20) // (S * L)))
+    sub = SI.shrink(cfg, n_canaries=n_can)
+    acts, refs, labels = O.generate_pipeline(O.desc_from_dict(sub), n_threads=n_threads)
+    return {"acts": acts, "refs": refs, "labels": labels, "S": S, "n": n_can, "L": L}
+
+
+def oracle_pass(sample, n_threads):
+    """One pass of the oracle verifier over the sample: drift scores + AUROC."""
+    from oracle import oracle as O
+    sc = O.drift_scores(sample["acts"], sample["refs"], sample["S"], sample["n"],
+                        n_threads=n_threads)
+    O.auroc(sc[0].astype(np.float32)[None], sample["labels"][None])
+
+
+def oracle_describe(sample, passes, seconds):
+    S, n, L = sample["S"], sample["n"], sample["L"]
+    e = S * n * L
+    return (f"{S} stages x {n} canaries x {L} elements ({e} elements, "
+            f"{e * BYTES_PER_ELEMENT / 1e9:.2f} GB) of the workload, generated by the oracle; "
+            f"drift scores + AUROC in fp64, {passes} passes in {seconds:.1f} s")
+
+
+def oracle_baseline(cfg, n_threads, seconds):
+    """Time the oracle on the sample, repeating passes until `seconds` elapse."""
+    sample = oracle_prepare(cfg, n_threads)
+    elems = sample["S"] * sample["n"] * sample["L"]
+    passes, t0 = 0, time.perf_counter()
+    while True:
+        oracle_pass(sample, n_threads)
+        passes += 1
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return {"value": elems * passes / el, "unit": "elements/s", "cores": n_threads,
+            "kind": "oracle", "sample": oracle_describe(sample, passes, el)}
+
+
+def run_reference(args, ranks: Ranks):
+    """The reference arm: the fp64 CPU oracle, one pass over the bounded
+    sample per step, on all host cores."""
+    if ranks.rank != 0:
+        return
+    cfg = WORKLOADS[args.workload]
+    from oracle import oracle as O
+    O.build()
+    threads = O.max_threads()
+    sample = oracle_prepare(cfg, threads)
+    elems = sample["S"] * sample["n"] * sample["L"]
+    for _ in range(args.warmup):
+        oracle_pass(sample, threads)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_pass(sample, threads)
+        times.append(time.perf_counter() - t0)
+    value = elems / statistics.median(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "elements/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000 * statistics.mean(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD_NAMES[args.workload],
+                   "sample": oracle_describe(sample, args.steps, sum(times))},
+        "cpu_baseline": {"value": value, "unit": "elements/s", "cores": threads,
+                         "kind": "oracle", "sample": oracle_describe(sample, args.steps, sum(times))},
+        "e2e": {"value": value, "unit": "elements/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args, ranks: Ranks):
+    import torch
+    import paper_2607_19490_gb300 as cg
+
+    if not torch.cuda.is_available():
+        raise RuntimeError("bench.py needs a CUDA device (no CPU fallback)")
+    torch.cuda.set_device(ranks.local)
+    cg.build()
+    cfg = rank_config(WORKLOADS[args.workload], ranks.rank)
+    S, N, T, d = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"], cfg["hidden"]
+    L = T * d
+    E = S * N * L
+    dev = torch.device("cuda", ranks.local)
+    stream = torch.cuda.current_stream()
+
+    # ---- resident inputs: materialised on the device by the generator
+    desc = cg.PipelineDesc.from_config(cfg)
+    acts = torch.empty((S, N, L), dtype=torch.float16, device=dev)
+    refs = torch.empty((S, N, L), dtype=torch.float32, device=dev)
+    labels = torch.empty((1, N, S), dtype=torch.int8, device=dev)
+    gws = torch.empty(cg.cg_generate_workspace_size(desc), dtype=torch.uint8, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    gen_ms = []
+    for i in range(2):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        cg.cg_generate_pipeline(desc, acts, refs, labels[0], gws, status=status)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        gen_ms.append(e0.elapsed_time(e1))
+    del gws
+
+    scores = torch.empty((3, 1, N, S), dtype=torch.float32, device=dev)
+    dws = torch.empty(cg.cg_drift_workspace_size(S, N, L), dtype=torch.uint8, device=dev)
+    ctrl = torch.empty((1, N, S), dtype=torch.int8, device=dev)
+    outs = {k: torch.empty((1, N), dtype=torch.int64, device=dev) for k in ("u2", "gt", "eq")}
+    outs_c = {k: torch.empty((1, N), dtype=torch.int64, device=dev) for k in ("u2", "gt", "eq")}
+    auroc = torch.empty((2,), dtype=torch.float64, device=dev)
+    launches_per_step = 5          # drift partial + finalize, control labels, 2 x AUROC
+
+    def step(i, ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        cg.cg_drift_scores(acts, refs, S, N, scores=scores, stat_stride=N * S, ws=dws,
+                           status=status)
+        if ev is not None:
+            ev[1].record(stream)
+        cg.cg_make_control_labels(labels, seed=1000 + i, ctrl=ctrl, status=status)
+        rel = scores[0]
+        cg.cg_auroc(rel, labels, u2=outs["u2"], gt=outs["gt"], eq=outs["eq"], auroc=auroc[0:1],
+                    status=status)
+        cg.cg_auroc(rel, ctrl, u2=outs_c["u2"], gt=outs_c["gt"], eq=outs_c["eq"],
+                    auroc=auroc[1:2], status=status)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    drift_events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                    for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(ranks.local)
+    clocks.start()
+    time.sleep(0.3)
+    ranks.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(args.warmup + i, drift_events[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    clk = clocks.stop()
+    total_ms = ranks.max(t_start.elapsed_time(t_end))
+    drift_ms = [a.elapsed_time(b) for a, b in drift_events]
+    st, word = cg.cg_read_status(status)
+    if st != 0:
+        raise RuntimeError(f"device status {word} after the timed steps")
+    auroc_true, auroc_ctrl = auroc.cpu().tolist()
+
+    total_elems = ranks.sum(float(E)) * args.steps
+    value = total_elems / (total_ms / 1e3)
+    peak, peak_kind = measured_peaks()
+    drift_avg_ms = statistics.mean(drift_ms)
+    achieved = E * BYTES_PER_ELEMENT / (drift_avg_ms / 1e3) / 1e9
+    traffic = recorded_traffic("drift.cu", f"drift_partial_kernel_{args.workload}.txt")
+
+    # ---- AUROC batches (configs/s): the factorial batch and a stress batch
+    auroc_rates = auroc_batches(cg, torch, dev, stream)
+
+    # ---- end to end with host buffers
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks)
+    del acts, refs
+    torch.cuda.empty_cache()
+
+    cpu = None
+    if ranks.rank == 0 and ranks.world == 1 and not args.no_cpu_baseline:
+        from oracle import oracle as O
+        cpu = oracle_baseline(WORKLOADS[args.workload], O.max_threads(), args.cpu_seconds)
+
+    if ranks.rank != 0:
+        return
+    gen_best = min(gen_ms)
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "elements/s",
+        "n_gpus": ranks.world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": total_ms / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": WORKLOAD_NAMES[args.workload], "n_shards": S, "hidden": d,
+            "n_canaries": N, "tokens": T, "elements_per_step": E,
+            "bytes_read_per_step": E * BYTES_PER_ELEMENT,
+            "l2": f"inputs {E * BYTES_PER_ELEMENT / 1e9:.1f} GB per step, larger than the "
+                  f"{L2_BYTES / 2**20:.0f} MB L2; no flush",
+            "step": "drift scores (2 kernels) + control labels + AUROC true and control",
+        },
+        "roofline": {
+            "kernel": "drift_partial_kernel (+ drift_finalize_kernel inside the same events)",
+            "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+            "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
+            "traffic": traffic,
+            "algorithmic_bytes_per_launch": E * BYTES_PER_ELEMENT,
+            "launch_ms_mean": drift_avg_ms, "launch_ms_min": min(drift_ms),
+        },
+        "auroc": {"true_labels": auroc_true, "control": auroc_ctrl, **auroc_rates},
+        "generate": {
+            "ms": gen_best, "elements_per_s": E / (gen_best / 1e3),
+            "write_GBps": E * BYTES_PER_ELEMENT / (gen_best / 1e3) / 1e9,
+        },
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def auroc_batches(cg, torch, dev, stream):
+    out = {}
+    g = torch.Generator(device=dev)
+    g.manual_seed(7)
+    for name, C, N, S in (("factorial_batch", 324, 64, 16), ("stress_batch", 65536, 64, 16)):
+        scores = torch.rand((C, N, S), generator=g, device=dev, dtype=torch.float32)
+        labels = torch.zeros((C, N, S), dtype=torch.int8, device=dev)
+        labels[:, :, 0] = 1
+        res = {k: torch.empty((C, N), dtype=torch.int64, device=dev) for k in ("u2",)}
+        au = torch.empty((C,), dtype=torch.float64, device=dev)
+        for _ in range(3):
+            cg.cg_auroc(scores, labels, u2=res["u2"], auroc=au, want_counts=False)
+        reps = 20
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            cg.cg_auroc(scores, labels, u2=res["u2"], auroc=au, want_counts=False)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        out[f"{name}_configs_per_s"] = C / (ms / 1e3)
+        out[f"{name}_ms"] = ms
+        del scores, labels
+    return out
+
+
+def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
+    """The same step with the inputs in pinned host memory: H2D copies of the
+    live activations and references, drift, control, AUROC, D2H of the scores
+    and A-hat, every step."""
+    h_acts = torch.empty(acts.shape, dtype=acts.dtype, pin_memory=True)
+    h_refs = torch.empty(refs.shape, dtype=refs.dtype, pin_memory=True)
+    h_acts.copy_(acts)
+    h_refs.copy_(refs)
+    h_scores = torch.empty((3, N, S), dtype=torch.float32, pin_memory=True)
+    h_auroc = torch.empty((2,), dtype=torch.float64, pin_memory=True)
+    scores = torch.empty((3, N, S), dtype=torch.float32, device=dev)
+    dws = torch.empty(cg.cg_drift_workspace_size(S, N, L), dtype=torch.uint8, device=dev)
+    ctrl = torch.empty_like(labels)
+    auroc = torch.empty((2,), dtype=torch.float64, device=dev)
+
+    def step(i):
+        acts.copy_(h_acts, non_blocking=True)
+        refs.copy_(h_refs, non_blocking=True)
+        cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=dws)
+        cg.cg_make_control_labels(labels, seed=5000 + i, ctrl=ctrl)
+        cg.cg_auroc(scores[0][None], labels, auroc=auroc[0:1], want_counts=False)
+        cg.cg_auroc(scores[0][None], ctrl, auroc=auroc[1:2], want_counts=False)
+        h_scores.copy_(scores, non_blocking=True)
+        h_auroc.copy_(auroc, non_blocking=True)
+
+    step(0)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(args.e2e_steps):
+        step(i + 1)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = ranks.max(e0.elapsed_time(e1)) / args.e2e_steps
+    elems = ranks.sum(float(S * N * L))
+    h2d = acts.numel() * acts.element_size() + refs.numel() * refs.element_size()
+    d2h = h_scores.numel() * 4 + h_auroc.numel() * 8
+    del h_acts, h_refs
+    return {"value": elems / (ms / 1e3), "unit": "elements/s", "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "ms_per_step": ms, "steps": args.e2e_steps,
+            "h2d_GBps": h2d / (ms / 1e3) / 1e9}
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    ranks = Ranks()
+    if args.impl == "reference":
+        if ranks.world > 1 and ranks.rank != 0:
+            return 0
+        run_reference(args, ranks)
+        return 0
+    ranks.init("nccl")
+    try:
+        run_ours(args, ranks)
+    finally:
+        ranks.close()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,223 @@
+/*
+ * canary_guard.h -- C ABI of the GB300 (sm_103a) canary-trap hot path.
+ *
+ * The library implements the verifier-side hot path of arxiv 2607.19490,
+ * "Integrity of peer-to-peer distributed LLM inference under malicious
+ * nodes":
+ *   - a synthetic k-stage pipeline: fp32 hop references and fp16 live
+ *     activations, benign (Eq. 2) or tampered (Eq. 3, Sec. 3.2);
+ *   - the drift scores of every (stage, canary) pair: the relative-L2
+ *     mismatch (Eq. 4), the max-abs deviation and the cosine mismatch of the
+ *     cosine-metric ablation (Sec. 4.4);
+ *   - the per-canary AUROC (Eq. 5) as exact Mann-Whitney counts, its mean
+ *     over canaries (Eq. 6) and the scrambled-label control (Sec. 4.5).
+ *
+ * Conventions shared by every entry point:
+ *   - Every buffer argument named d_* is caller-owned device memory; h_*
+ *     is host memory.  The library allocates no device memory, creates no
+ *     stream and never synchronises, except cg_read_status.
+ *   - Calls are asynchronous and ordered on `stream` (a cudaStream_t; NULL
+ *     is the legacy default stream).
+ *   - All arguments are validated on the host before any launch; a rejected
+ *     call launches nothing and returns the error.  CG_ERR_CUDA reports a
+ *     launch error (the CUDA error is left for the caller to inspect).
+ *   - Conditions only the device can see (a NaN score, a control canary
+ *     without a benign stage, a bounded wait that gave up) are OR-ed as
+ *     CG_DEVFLAG_* bits into an optional caller-owned int32 device word
+ *     d_status (may be NULL).  cg_read_status synchronises the stream and
+ *     maps the word to a cg_status.
+ *   - Results are deterministic run to run on one GPU: fixed reduction
+ *     order, no floating-point atomics.
+ *   - fp16 tensors are passed as uint16_t binary16 bit patterns.
+ *   - Layouts: live activations and references are [S][N][T][d] row-major
+ *     (one (stage, canary) segment = T*d contiguous elements); drift
+ *     scores are [stat][N][S] with stat 0 = rel_l2, 1 = max_abs,
+ *     2 = cos_dev; labels and AUROC inputs are [C][N][S] per configuration.
+ */
+#ifndef CANARY_GUARD_H
+#define CANARY_GUARD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st *cg_stream_t;
+
+typedef enum {
+  CG_OK = 0,
+  CG_ERR_INVALID_ARG = 1,   /* a NULL, zero or out-of-range argument */
+  CG_ERR_ALIGNMENT = 2,     /* a device pointer below its required alignment */
+  CG_ERR_WORKSPACE = 3,     /* workspace missing or smaller than the size query */
+  CG_ERR_NAN_SCORE = 4,     /* a labelled score is NaN (device flag) */
+  CG_ERR_CUDA = 5,          /* a CUDA launch or runtime call failed */
+  CG_ERR_TIMEOUT = 6,       /* a bounded device wait gave up (device flag) */
+  CG_ERR_UNSUPPORTED = 7,   /* a size beyond what this build handles */
+  CG_ERR_NO_BENIGN = 8      /* a control canary had no benign stage (device flag) */
+} cg_status;
+
+/* Bits of the device status word. */
+#define CG_DEVFLAG_NAN_SCORE 1
+#define CG_DEVFLAG_TIMEOUT 2
+#define CG_DEVFLAG_NO_BENIGN 4
+
+/* Benign noise of a stage outside the malicious set (Eq. 2). */
+typedef enum {
+  CG_NOISE_MULT = 0,   /* h = fp16(a (1 + sigma_s z)): relative per-element noise */
+  CG_NOISE_PAPER = 1   /* h = fp16(a + sigma_s mu z), mu = ||a||_1 / (T d) (Eq. 2) */
+} cg_noise_model;
+
+/* Tamper applied by a malicious stage (Eq. 3 and the strategies of Sec. 3.2). */
+typedef enum {
+  CG_TAMPER_ADDITIVE = 0,          /* a + eps ||a||_F g / ||g||_F, eps = tamper_param */
+  CG_TAMPER_SIGNFLIP_CHANNELS = 1, /* negate max(1, round(p d)) channels, p = tamper_param */
+  CG_TAMPER_SIGNFLIP_FULL = 2,     /* -a */
+  CG_TAMPER_SCALE = 3              /* beta a, beta = tamper_param */
+} cg_tamper_kind;
+
+/*
+ * One synthetic pipeline configuration: k = n_shards stages of hidden size
+ * d, n canaries of T tokens (Sec. 3.1, Sec. 3.3), the malicious set M
+ * (Sec. 3.2), sigma_hw (Eq. 2) and the tamper parameter.  Random draws use
+ * Philox4x32-10 (Salmon et al., SC'11) keyed by `seed` with config_id in the
+ * counter, so every value is a pure function of the description.
+ */
+typedef struct {
+  uint32_t n_shards;             /* k >= 1 stages (shards), at most 1024 */
+  uint32_t hidden;               /* d >= 1 */
+  uint32_t n_canaries;           /* n >= 1 */
+  uint32_t tokens;               /* T >= 1; T * d < 2^34 */
+  const int32_t *malicious;      /* host array of n_malicious distinct 0-based stage ids */
+  uint32_t n_malicious;          /* c = |M|, 0 <= c < k */
+  int32_t noise;                 /* cg_noise_model */
+  float benign_sigma;            /* sigma_hw >= 0 */
+  float shard_sigma_lognormal;   /* lambda >= 0: sigma_s = sigma exp(lambda z_s); 0 = same sigma */
+  uint32_t n_outlier;            /* outlier channels per configuration, <= min(d, 256) */
+  float outlier_scale;           /* reference multiplier on outlier channels */
+  int32_t tamper;                /* cg_tamper_kind */
+  float tamper_param;            /* eps | channel fraction in (0, 1] | scale factor */
+  uint64_t seed;                 /* Philox key */
+  uint32_t config_id;            /* < 2^30; separates the draws of configurations */
+} cg_pipeline_desc;
+
+/* Human-readable name of a status code (static storage). */
+const char *cg_status_string(cg_status status);
+
+/* ABI version of this header (incremented on incompatible changes). */
+int cg_abi_version(void);
+
+/*
+ * Philox4x32-10 blocks first_block .. first_block + n_blocks - 1 with
+ * counter (block, c1, c2, c3) and key (seed lo, seed hi) (SC'11), written
+ * block-major to d_out (4 * n_blocks words, 16-byte aligned).  This is the
+ * stream every generator draw is taken from (seed semantics, Sec. 4.4).
+ */
+cg_status cg_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                          uint32_t first_block, uint32_t n_blocks,
+                          uint32_t *d_out, cg_stream_t stream);
+
+/*
+ * The Box-Muller normals of the same blocks (the Gaussians of Eq. 2 and of
+ * the Gaussian tamper, Sec. 3.2): per block, (x0, x1) -> normals 0, 1 and
+ * (x2, x3) -> normals 2, 3 with u1 = ((x >> 8) + 1) 2^-24,
+ * u2 = (x >> 8) 2^-24, z = sqrt(-2 ln u1) (cos, sin)(2 pi u2), in fp32.
+ * d_out: 4 * n_blocks floats, 16-byte aligned.
+ */
+cg_status cg_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                            uint32_t first_block, uint32_t n_blocks,
+                            float *d_out, cg_stream_t stream);
+
+/* Workspace bytes cg_generate_pipeline needs for `desc`. */
+cg_status cg_generate_workspace_size(const cg_pipeline_desc *desc, size_t *bytes);
+
+/*
+ * Materialise one pipeline configuration (Eq. 1-3 stand-in, Sec. 3.3):
+ *   d_refs   fp32 [S][N][T][d]  reference a (stored fp32 references)
+ *   d_acts   fp16 [S][N][T][d]  live h: benign stages per `noise` (Eq. 2),
+ *                               malicious stages per `tamper` (Eq. 3)
+ *   d_labels int8 [N][S] or NULL: 1 on malicious stages, else 0
+ *   d_ws     workspace of ws_bytes >= cg_generate_workspace_size, 16-byte
+ *            aligned; its contents are scratch.
+ * d_acts and d_refs must be 16-byte aligned.  A distinct-channel draw that
+ * exhausts its draw cap (not expected for valid descriptions) raises
+ * CG_DEVFLAG_TIMEOUT in d_status.
+ */
+cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts,
+                               float *d_refs, int8_t *d_labels, void *d_ws,
+                               size_t ws_bytes, int32_t *d_status,
+                               cg_stream_t stream);
+
+/* Workspace bytes cg_drift_scores needs for S * N segments of seg_len. */
+cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
+                                  uint64_t seg_len, size_t *bytes);
+
+/*
+ * Drift scores of every (stage s, canary n) segment (Eq. 4 and Sec. 4.4):
+ *   rel_l2  = ||h - a||_F / ||a||_F (0 if both are zero, +inf if only a is)
+ *   max_abs = max |h - a|           (computed in fp32, exact)
+ *   cos_dev = 1 - h.a / (||h|| ||a||) (0 when either norm is zero)
+ * d_acts fp16 and d_refs fp32 are [S][N][seg_len], 16-byte aligned; any
+ * seg_len >= 1 (ragged tails handled).  Scores are written to
+ * d_scores[stat * stat_stride + n * S + s] (stat_stride >= N * S; pass
+ * N * S for a dense [3][N][S] block).  Each element of d_acts and d_refs is
+ * read once from HBM.  d_ws: >= cg_drift_workspace_size bytes, 16-byte
+ * aligned, scratch.
+ */
+cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
+                          uint32_t n_shards, uint32_t n_canaries,
+                          uint64_t seg_len, float *d_scores,
+                          uint64_t stat_stride, void *d_ws, size_t ws_bytes,
+                          int32_t *d_status, cg_stream_t stream);
+
+/*
+ * Scrambled-label negative control (Sec. 4.5).  For every configuration c
+ * and canary n, a stage j* is drawn uniformly from the stages labelled 0 in
+ * d_labels (ascending order; Philox aux stream 4 with config id
+ * config_id0 + c) and labelled 1; the stages labelled 1 in d_labels become
+ * -1 (left out); the other benign stages stay 0.
+ * d_labels, d_ctrl: int8 [C][N][S].  A canary with no benign stage gets no
+ * j* and raises CG_DEVFLAG_NO_BENIGN.
+ */
+cg_status cg_make_control_labels(const int8_t *d_labels, uint32_t n_configs,
+                                 uint32_t n_canaries, uint32_t n_shards,
+                                 uint64_t seed, uint32_t config_id0,
+                                 int8_t *d_ctrl, int32_t *d_status,
+                                 cg_stream_t stream);
+
+/*
+ * Exact Mann-Whitney counts and AUROC (Eq. 5, Eq. 6).
+ *   d_scores fp32 [C][N][S] (one statistic), d_labels int8 [C][N][S]:
+ *   1 = malicious, 0 = benign, anything else = left out.
+ * Per (c, n): gt = #{(i, j): label 1, label 0, m_i > m_j},
+ *             eq = #{same pairs with m_i == m_j},
+ *             d_u2[c][n] = 2 gt + eq (twice U; ties count one half).
+ * Per c: d_auroc[c] = mean over canaries with at least one pair of
+ * U / (c_t b_t); when every such canary has the same pair count P this is
+ * sum(u2) / (2 P N_valid), one fp64 division of exact integers; otherwise
+ * the per-canary ratios are added in canary order.  NaN when no canary has
+ * a pair.  d_u2 and d_auroc are required; d_gt, d_eq may be NULL.  A NaN
+ * labelled score raises CG_DEVFLAG_NAN_SCORE (its comparisons count as
+ * neither greater nor equal).  S up to 1024.
+ */
+cg_status cg_auroc(const float *d_scores, const int8_t *d_labels,
+                   uint32_t n_configs, uint32_t n_canaries, uint32_t n_shards,
+                   int64_t *d_u2, int64_t *d_gt, int64_t *d_eq,
+                   double *d_auroc, int32_t *d_status, cg_stream_t stream);
+
+/*
+ * Synchronise `stream`, read the device status word and map it: 0 ->
+ * CG_OK, else the first of CG_ERR_TIMEOUT, CG_ERR_NAN_SCORE,
+ * CG_ERR_NO_BENIGN that is set.  The raw word goes to *h_word if non-NULL.
+ * The word is not cleared.
+ */
+cg_status cg_read_status(const int32_t *d_status, cg_stream_t stream,
+                         int32_t *h_word);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CANARY_GUARD_H */

@@ -1,0 +1,293 @@
+"""GB300-native canary-trap hot path (arxiv 2607.19490): a thin ctypes binding
+over ``libcanary_guard.so`` (declared in ``include/canary_guard.h``).
+
+Functions keep the C names (``cg_generate_pipeline``, ``cg_drift_scores``,
+``cg_auroc``, ...).  They only marshal torch CUDA tensors into device
+pointers and the current stream; every step of the path runs in the
+library's CUDA kernels.  There is no CPU fallback: without the built library
+(``paper_2607_19490_gb300.build.build()``) or without a CUDA device every
+call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+from .build import LIB_PATH, build  # noqa: F401
+
+__all__ = [
+    "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
+    "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
+    "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
+    "cg_make_control_labels", "cg_auroc", "cg_read_status",
+    "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
+    "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
+]
+
+CG_OK = 0
+STATUS_NAMES = {0: "CG_OK", 1: "CG_ERR_INVALID_ARG", 2: "CG_ERR_ALIGNMENT", 3: "CG_ERR_WORKSPACE",
+                4: "CG_ERR_NAN_SCORE", 5: "CG_ERR_CUDA", 6: "CG_ERR_TIMEOUT",
+                7: "CG_ERR_UNSUPPORTED", 8: "CG_ERR_NO_BENIGN"}
+NOISE_MULT, NOISE_PAPER = 0, 1
+TAMPER_ADDITIVE, TAMPER_SIGNFLIP_CHANNELS, TAMPER_SIGNFLIP_FULL, TAMPER_SCALE = 0, 1, 2, 3
+DEVFLAG_NAN_SCORE, DEVFLAG_TIMEOUT, DEVFLAG_NO_BENIGN = 1, 2, 4
+
+
+class CgError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {STATUS_NAMES.get(status, status)}")
+
+
+class PipelineDesc(ctypes.Structure):
+    """Mirror of ``cg_pipeline_desc``."""
+    _fields_ = [
+        ("n_shards", ctypes.c_uint32), ("hidden", ctypes.c_uint32),
+        ("n_canaries", ctypes.c_uint32), ("tokens", ctypes.c_uint32),
+        ("malicious", ctypes.POINTER(ctypes.c_int32)), ("n_malicious", ctypes.c_uint32),
+        ("noise", ctypes.c_int32), ("benign_sigma", ctypes.c_float),
+        ("shard_sigma_lognormal", ctypes.c_float), ("n_outlier", ctypes.c_uint32),
+        ("outlier_scale", ctypes.c_float), ("tamper", ctypes.c_int32),
+        ("tamper_param", ctypes.c_float), ("seed", ctypes.c_uint64),
+        ("config_id", ctypes.c_uint32),
+    ]
+
+    @classmethod
+    def from_config(cls, cfg: dict) -> "PipelineDesc":
+        mal = (ctypes.c_int32 * max(1, len(cfg["malicious"])))(*cfg["malicious"])
+        d = cls(cfg["n_shards"], cfg["hidden"], cfg["n_canaries"], cfg["tokens"],
+                ctypes.cast(mal, ctypes.POINTER(ctypes.c_int32)), len(cfg["malicious"]),
+                cfg["noise"], cfg["benign_sigma"], cfg.get("shard_sigma_lognormal", 0.0),
+                cfg.get("n_outlier", 0), cfg.get("outlier_scale", 20.0), cfg["tamper"],
+                cfg["tamper_param"], cfg["seed"], cfg.get("config_id", 0))
+        d._keep = mal
+        return d
+
+    @property
+    def seg_len(self) -> int:
+        return self.tokens * self.hidden
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def load() -> ctypes.CDLL:
+    """Load the built library (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build the CUDA library first "
+                "(python -c 'import __graft_entry__ as g; g.build()'); there is no CPU fallback")
+        L = ctypes.CDLL(LIB_PATH)
+        P, u32, u64, i32, sz = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int32, ctypes.c_size_t
+        sigs = {
+            "cg_status_string": ([ctypes.c_int], ctypes.c_char_p),
+            "cg_abi_version": ([], ctypes.c_int),
+            "cg_philox_words": ([u64, u32, u32, u32, u32, u32, P, P], ctypes.c_int),
+            "cg_philox_normals": ([u64, u32, u32, u32, u32, u32, P, P], ctypes.c_int),
+            "cg_generate_workspace_size": ([ctypes.POINTER(PipelineDesc), ctypes.POINTER(sz)], ctypes.c_int),
+            "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
+            "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
+            "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
+            "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
+            "cg_auroc": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
+            "cg_read_status": ([P, P, ctypes.POINTER(i32)], ctypes.c_int),
+        }
+        for name, (args, res) in sigs.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+        return _lib
+
+
+# --------------------------------------------------------------------------- helpers
+
+def _torch():
+    import torch
+    return torch
+
+
+def _check(status: int, where: str):
+    if status != CG_OK:
+        raise CgError(status, where)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _cuda(t, name, dtypes):
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if t.dtype not in dtypes:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+
+
+def _stream(stream):
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def cg_status_string(status: int) -> str:
+    return load().cg_status_string(status).decode()
+
+
+def cg_abi_version() -> int:
+    return int(load().cg_abi_version())
+
+
+# --------------------------------------------------------------------------- entry points
+
+def cg_philox_words(seed, c1, c2, c3, first_block, n_blocks, out=None, stream=None):
+    """Philox4x32-10 blocks as an int32 tensor [n_blocks, 4] (bit patterns of uint32)."""
+    torch = _torch()
+    if out is None:
+        out = torch.empty((n_blocks, 4), dtype=torch.int32, device="cuda")
+    _cuda(out, "out", (torch.int32,))
+    _check(load().cg_philox_words(seed, c1, c2, c3, first_block, n_blocks, _ptr(out),
+                                  _stream(stream)), "cg_philox_words")
+    return out
+
+
+def cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, out=None, stream=None):
+    torch = _torch()
+    if out is None:
+        out = torch.empty((n_blocks, 4), dtype=torch.float32, device="cuda")
+    _cuda(out, "out", (torch.float32,))
+    _check(load().cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, _ptr(out),
+                                    _stream(stream)), "cg_philox_normals")
+    return out
+
+
+def cg_generate_workspace_size(desc: PipelineDesc) -> int:
+    n = ctypes.c_size_t()
+    _check(load().cg_generate_workspace_size(ctypes.byref(desc), ctypes.byref(n)),
+           "cg_generate_workspace_size")
+    return n.value
+
+
+def cg_generate_pipeline(desc: PipelineDesc, acts=None, refs=None, labels=None, ws=None,
+                         status=None, stream=None, want_labels=True):
+    """Materialise one configuration; returns (acts fp16, refs fp32, labels int8 or None),
+    acts/refs shaped [S][N][T*d], labels [N][S]."""
+    torch = _torch()
+    S, N, L = desc.n_shards, desc.n_canaries, desc.seg_len
+    if acts is None:
+        acts = torch.empty((S, N, L), dtype=torch.float16, device="cuda")
+    if refs is None:
+        refs = torch.empty((S, N, L), dtype=torch.float32, device="cuda")
+    if labels is None and want_labels:
+        labels = torch.empty((N, S), dtype=torch.int8, device="cuda")
+    need = cg_generate_workspace_size(desc)
+    if ws is None:
+        ws = torch.empty(need, dtype=torch.uint8, device="cuda")
+    _cuda(acts, "acts", (torch.float16,))
+    _cuda(refs, "refs", (torch.float32,))
+    _cuda(labels, "labels", (torch.int8,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    if acts.numel() != S * N * L or refs.numel() != S * N * L:
+        raise ValueError("acts/refs must hold S*N*T*d elements")
+    if labels is not None and labels.numel() != N * S:
+        raise ValueError("labels must hold N*S elements")
+    _check(load().cg_generate_pipeline(ctypes.byref(desc), _ptr(acts), _ptr(refs), _ptr(labels),
+                                       _ptr(ws), ws.numel(), _ptr(status), _stream(stream)),
+           "cg_generate_pipeline")
+    return acts, refs, labels
+
+
+def cg_drift_workspace_size(n_shards, n_canaries, seg_len) -> int:
+    n = ctypes.c_size_t()
+    _check(load().cg_drift_workspace_size(n_shards, n_canaries, seg_len, ctypes.byref(n)),
+           "cg_drift_workspace_size")
+    return n.value
+
+
+def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=None, ws=None,
+                    status=None, stream=None):
+    """Drift scores [3][N][S] (rel_l2, max_abs, cos_dev) of acts fp16 / refs fp32 [S][N][L]."""
+    torch = _torch()
+    _cuda(acts, "acts", (torch.float16,))
+    _cuda(refs, "refs", (torch.float32,))
+    n_seg = n_shards * n_canaries
+    if acts.numel() != refs.numel() or acts.numel() % n_seg:
+        raise ValueError("acts and refs must both hold S*N*L elements")
+    seg_len = acts.numel() // n_seg
+    if scores is None:
+        scores = torch.empty((3, n_canaries, n_shards), dtype=torch.float32, device=acts.device)
+        stat_stride = n_seg
+    if stat_stride is None:
+        stat_stride = n_seg
+    if ws is None:
+        ws = torch.empty(cg_drift_workspace_size(n_shards, n_canaries, seg_len), dtype=torch.uint8,
+                         device=acts.device)
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
+                                  _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
+                                  _stream(stream)), "cg_drift_scores")
+    return scores
+
+
+def cg_make_control_labels(labels, seed, config_id0=0, ctrl=None, status=None, stream=None):
+    """Scrambled-label control for labels int8 [C][N][S]."""
+    torch = _torch()
+    _cuda(labels, "labels", (torch.int8,))
+    C, N, S = labels.shape
+    if ctrl is None:
+        ctrl = torch.empty_like(labels)
+    _cuda(ctrl, "ctrl", (torch.int8,))
+    _cuda(status, "status", (torch.int32,))
+    _check(load().cg_make_control_labels(_ptr(labels), C, N, S, seed, config_id0, _ptr(ctrl),
+                                         _ptr(status), _stream(stream)), "cg_make_control_labels")
+    return ctrl
+
+
+def cg_auroc(scores, labels, u2=None, gt=None, eq=None, auroc=None, status=None, stream=None,
+             want_counts=True):
+    """Mann-Whitney counts and AUROC of scores fp32 / labels int8 [C][N][S].
+
+    Returns dict(u2, gt, eq, auroc) of device tensors (gt/eq None unless wanted)."""
+    torch = _torch()
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(labels, "labels", (torch.int8,))
+    if scores.shape != labels.shape or scores.dim() != 3:
+        raise ValueError("scores and labels must both be [C][N][S]")
+    C, N, S = scores.shape
+    dev = scores.device
+    if u2 is None:
+        u2 = torch.empty((C, N), dtype=torch.int64, device=dev)
+    if want_counts and gt is None:
+        gt = torch.empty((C, N), dtype=torch.int64, device=dev)
+    if want_counts and eq is None:
+        eq = torch.empty((C, N), dtype=torch.int64, device=dev)
+    if auroc is None:
+        auroc = torch.empty((C,), dtype=torch.float64, device=dev)
+    for t, n in ((u2, "u2"), (gt, "gt"), (eq, "eq")):
+        _cuda(t, n, (torch.int64,))
+    _cuda(auroc, "auroc", (torch.float64,))
+    _cuda(status, "status", (torch.int32,))
+    _check(load().cg_auroc(_ptr(scores), _ptr(labels), C, N, S, _ptr(u2), _ptr(gt), _ptr(eq),
+                           _ptr(auroc), _ptr(status), _stream(stream)), "cg_auroc")
+    return {"u2": u2, "gt": gt, "eq": eq, "auroc": auroc}
+
+
+def cg_read_status(status, stream=None):
+    """Synchronise and read a device status word: returns (cg_status, raw word)."""
+    torch = _torch()
+    _cuda(status, "status", (torch.int32,))
+    word = ctypes.c_int32()
+    st = load().cg_read_status(_ptr(status), _stream(stream), ctypes.byref(word))
+    return st, word.value

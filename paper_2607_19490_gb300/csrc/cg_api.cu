@@ -1,0 +1,235 @@
+// cg_api.cu -- the C ABI declared in include/canary_guard.h: argument
+// validation on the host, workspace sizing and kernel dispatch.  No entry
+// point allocates device memory or synchronises (except cg_read_status).
+#include <math.h>
+#include <mutex>
+#include <string.h>
+
+#include "cg_internal.h"
+
+namespace cg {
+
+int drift_occupancy();
+int gen_occupancy();
+
+bool device_info(DeviceInfo *out) {
+  static std::mutex mu;
+  static DeviceInfo cache[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return false;
+  std::lock_guard<std::mutex> lock(mu);
+  if (dev < 64 && cache[dev].device == dev) {
+    *out = cache[dev];
+    return true;
+  }
+  DeviceInfo info;
+  info.device = dev;
+  if (cudaDeviceGetAttribute(&info.sm_count, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  info.drift_blocks_per_sm = drift_occupancy();
+  info.gen_blocks_per_sm = gen_occupancy();
+  if (info.drift_blocks_per_sm < 1 || info.gen_blocks_per_sm < 1) return false;
+  if (dev < 64) cache[dev] = info;
+  *out = info;
+  return true;
+}
+
+}  // namespace cg
+
+namespace {
+
+inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+inline cg_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CG_OK : CG_ERR_CUDA; }
+
+cg_status check_desc(const cg_pipeline_desc *d) {
+  if (!d) return CG_ERR_INVALID_ARG;
+  if (d->n_shards < 1 || d->hidden < 1 || d->n_canaries < 1 || d->tokens < 1)
+    return CG_ERR_INVALID_ARG;
+  if (d->n_shards > cg::kMaxShards) return CG_ERR_UNSUPPORTED;
+  const uint64_t L = (uint64_t)d->tokens * d->hidden;
+  if (L >= (1ull << 34)) return CG_ERR_UNSUPPORTED;
+  if ((uint64_t)d->n_shards * d->n_canaries >= (1ull << 32)) return CG_ERR_UNSUPPORTED;
+  if (d->config_id >= (1u << 30)) return CG_ERR_INVALID_ARG;
+  if (d->n_malicious >= d->n_shards) return CG_ERR_INVALID_ARG;
+  if (d->n_malicious > 0 && !d->malicious) return CG_ERR_INVALID_ARG;
+  if (d->noise != CG_NOISE_MULT && d->noise != CG_NOISE_PAPER) return CG_ERR_INVALID_ARG;
+  if (d->tamper < CG_TAMPER_ADDITIVE || d->tamper > CG_TAMPER_SCALE) return CG_ERR_INVALID_ARG;
+  if (d->n_outlier > d->hidden) return CG_ERR_INVALID_ARG;
+  if (d->n_outlier > cg::kMaxOutliers) return CG_ERR_UNSUPPORTED;
+  if (!isfinite(d->benign_sigma) || d->benign_sigma < 0.f) return CG_ERR_INVALID_ARG;
+  if (!isfinite(d->shard_sigma_lognormal) || d->shard_sigma_lognormal < 0.f)
+    return CG_ERR_INVALID_ARG;
+  if (!isfinite(d->outlier_scale) || !isfinite(d->tamper_param)) return CG_ERR_INVALID_ARG;
+  if (d->tamper == CG_TAMPER_SIGNFLIP_CHANNELS &&
+      !(d->tamper_param > 0.f && d->tamper_param <= 1.f))
+    return CG_ERR_INVALID_ARG;
+  for (uint32_t i = 0; i < d->n_malicious; ++i) {
+    const int32_t s = d->malicious[i];
+    if (s < 0 || (uint32_t)s >= d->n_shards) return CG_ERR_INVALID_ARG;
+    for (uint32_t j = 0; j < i; ++j)
+      if (d->malicious[j] == s) return CG_ERR_INVALID_ARG;
+  }
+  return CG_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *cg_status_string(cg_status s) {
+  switch (s) {
+    case CG_OK: return "CG_OK";
+    case CG_ERR_INVALID_ARG: return "CG_ERR_INVALID_ARG: invalid argument";
+    case CG_ERR_ALIGNMENT: return "CG_ERR_ALIGNMENT: device pointer misaligned";
+    case CG_ERR_WORKSPACE: return "CG_ERR_WORKSPACE: workspace missing or too small";
+    case CG_ERR_NAN_SCORE: return "CG_ERR_NAN_SCORE: a labelled score is NaN";
+    case CG_ERR_CUDA: return "CG_ERR_CUDA: CUDA launch or runtime error";
+    case CG_ERR_TIMEOUT: return "CG_ERR_TIMEOUT: a bounded device wait gave up";
+    case CG_ERR_UNSUPPORTED: return "CG_ERR_UNSUPPORTED: size beyond this build's limits";
+    case CG_ERR_NO_BENIGN: return "CG_ERR_NO_BENIGN: a control canary had no benign stage";
+  }
+  return "unknown cg_status";
+}
+
+int cg_abi_version(void) { return 1; }
+
+cg_status cg_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                          uint32_t first_block, uint32_t n_blocks, uint32_t *d_out,
+                          cg_stream_t stream) {
+  if (!d_out || n_blocks == 0) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_out, 16)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_philox_words(seed, c1, c2, c3, first_block, n_blocks, d_out,
+                                           (cudaStream_t)stream));
+}
+
+cg_status cg_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                            uint32_t first_block, uint32_t n_blocks, float *d_out,
+                            cg_stream_t stream) {
+  if (!d_out || n_blocks == 0) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_out, 16)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_philox_normals(seed, c1, c2, c3, first_block, n_blocks, d_out,
+                                             (cudaStream_t)stream));
+}
+
+cg_status cg_generate_workspace_size(const cg_pipeline_desc *desc, size_t *bytes) {
+  if (!bytes) return CG_ERR_INVALID_ARG;
+  cg_status st = check_desc(desc);
+  if (st != CG_OK) return st;
+  *bytes = cg::gen_layout(*desc).total;
+  return CG_OK;
+}
+
+cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts, float *d_refs,
+                               int8_t *d_labels, void *d_ws, size_t ws_bytes, int32_t *d_status,
+                               cg_stream_t stream) {
+  cg_status st = check_desc(desc);
+  if (st != CG_OK) return st;
+  if (!d_acts || !d_refs) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  const cg::GenLayout lay = cg::gen_layout(*desc);
+  if (!d_ws || ws_bytes < lay.total) return CG_ERR_WORKSPACE;
+  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
+
+  cg::GenParams p;
+  memset(&p, 0, sizeof(p));
+  p.seed = desc->seed;
+  p.S = desc->n_shards;
+  p.N = desc->n_canaries;
+  p.T = desc->tokens;
+  p.d = desc->hidden;
+  p.L = (uint64_t)desc->tokens * desc->hidden;
+  p.config_id = desc->config_id;
+  p.noise = desc->noise;
+  p.tamper = desc->tamper;
+  p.sigma = desc->benign_sigma;
+  p.lognormal = desc->shard_sigma_lognormal;
+  p.outlier_scale = desc->outlier_scale;
+  p.tamper_param = desc->tamper_param;
+  p.n_outlier = desc->n_outlier;
+  // max(1, round-half-up(p d)) flipped channels, evaluated in double
+  double r = floor((double)desc->tamper_param * (double)desc->hidden + 0.5);
+  uint32_t nf = r < 1.0 ? 1u : (r > (double)desc->hidden ? desc->hidden : (uint32_t)r);
+  p.n_flip = nf;
+  p.mask_words = lay.mask_words;
+  p.stat_chunks = lay.stat_chunks;
+  for (uint32_t i = 0; i < desc->n_malicious; ++i) {
+    const uint32_t s = (uint32_t)desc->malicious[i];
+    p.mal_bits[s >> 5] |= 1u << (s & 31);
+  }
+  return from_cuda(cg::launch_generate(p, d_acts, d_refs, d_labels, d_ws, lay, d_status,
+                                       (cudaStream_t)stream));
+}
+
+cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
+                                  size_t *bytes) {
+  if (!bytes || n_shards == 0 || n_canaries == 0 || seg_len == 0) return CG_ERR_INVALID_ARG;
+  *bytes = cg::drift_ws_bytes((uint64_t)n_shards * n_canaries, seg_len);
+  return CG_OK;
+}
+
+cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs, uint32_t n_shards,
+                          uint32_t n_canaries, uint64_t seg_len, float *d_scores,
+                          uint64_t stat_stride, void *d_ws, size_t ws_bytes, int32_t *d_status,
+                          cg_stream_t stream) {
+  if (!d_acts || !d_refs || !d_scores || n_shards == 0 || n_canaries == 0 || seg_len == 0)
+    return CG_ERR_INVALID_ARG;
+  const uint64_t n_seg = (uint64_t)n_shards * n_canaries;
+  if (stat_stride < n_seg) return CG_ERR_INVALID_ARG;
+  if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
+  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || !aligned(d_scores, 4) ||
+      (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  if (!d_ws || ws_bytes < cg::drift_ws_bytes(n_seg, seg_len)) return CG_ERR_WORKSPACE;
+  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
+  (void)d_status;   // the streaming path has no device-side failure mode
+  return from_cuda(cg::launch_drift(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores,
+                                    stat_stride, d_ws, (cudaStream_t)stream));
+}
+
+cg_status cg_make_control_labels(const int8_t *d_labels, uint32_t n_configs,
+                                 uint32_t n_canaries, uint32_t n_shards, uint64_t seed,
+                                 uint32_t config_id0, int8_t *d_ctrl, int32_t *d_status,
+                                 cg_stream_t stream) {
+  if (!d_labels || !d_ctrl || n_configs == 0 || n_canaries == 0 || n_shards == 0)
+    return CG_ERR_INVALID_ARG;
+  if ((uint64_t)config_id0 + n_configs > (1ull << 30)) return CG_ERR_INVALID_ARG;
+  if (n_canaries > (1u << 24)) return CG_ERR_UNSUPPORTED;
+  if ((uint64_t)n_configs * n_canaries * n_shards >= (1ull << 40)) return CG_ERR_UNSUPPORTED;
+  if (d_status && !aligned(d_status, 4)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_control_labels(d_labels, n_configs, n_canaries, n_shards, seed,
+                                             config_id0, d_ctrl, d_status,
+                                             (cudaStream_t)stream));
+}
+
+cg_status cg_auroc(const float *d_scores, const int8_t *d_labels, uint32_t n_configs,
+                   uint32_t n_canaries, uint32_t n_shards, int64_t *d_u2, int64_t *d_gt,
+                   int64_t *d_eq, double *d_auroc, int32_t *d_status, cg_stream_t stream) {
+  if (!d_scores || !d_labels || !d_u2 || !d_auroc || n_configs == 0 || n_canaries == 0 ||
+      n_shards == 0)
+    return CG_ERR_INVALID_ARG;
+  if (n_shards > cg::kMaxRankShards) return CG_ERR_UNSUPPORTED;
+  if ((uint64_t)n_configs * n_canaries * n_shards >= (1ull << 40)) return CG_ERR_UNSUPPORTED;
+  if (!aligned(d_scores, 4) || !aligned(d_u2, 8) || !aligned(d_auroc, 8) ||
+      (d_gt && !aligned(d_gt, 8)) || (d_eq && !aligned(d_eq, 8)) ||
+      (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_auroc(d_scores, d_labels, n_configs, n_canaries, n_shards, d_u2,
+                                    d_gt, d_eq, d_auroc, d_status, (cudaStream_t)stream));
+}
+
+cg_status cg_read_status(const int32_t *d_status, cg_stream_t stream, int32_t *h_word) {
+  if (!d_status) return CG_ERR_INVALID_ARG;
+  int32_t w = 0;
+  cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+  if (e == cudaSuccess) e = cudaMemcpy(&w, d_status, sizeof(w), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return CG_ERR_CUDA;
+  if (h_word) *h_word = w;
+  if (w & CG_DEVFLAG_TIMEOUT) return CG_ERR_TIMEOUT;
+  if (w & CG_DEVFLAG_NAN_SCORE) return CG_ERR_NAN_SCORE;
+  if (w & CG_DEVFLAG_NO_BENIGN) return CG_ERR_NO_BENIGN;
+  return CG_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,85 @@
+// cg_internal.h -- launchers and workspace layouts shared by the library's
+// translation units (host side).  Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/canary_guard.h"
+
+namespace cg {
+
+// ---------------------------------------------------------------- device info
+struct DeviceInfo {
+  int device = -1;
+  int sm_count = 0;
+  int drift_blocks_per_sm = 0;
+  int gen_blocks_per_sm = 0;
+};
+// Cached per current device; returns false on a CUDA error.
+bool device_info(DeviceInfo *out);
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// ---------------------------------------------------------------- drift
+// A work item is a chunk of at most kDriftChunk elements of one segment.
+constexpr uint32_t kDriftChunk = 16384;
+constexpr int kDriftThreads = 256;
+constexpr size_t kDriftHeader = 256;   // reserved bytes at the start of the workspace
+
+inline uint64_t drift_chunks_per_seg(uint64_t seg_len) {
+  return (seg_len + kDriftChunk - 1) / kDriftChunk;
+}
+inline size_t drift_ws_bytes(uint64_t n_segments, uint64_t seg_len) {
+  return kDriftHeader + align_up((size_t)(n_segments * drift_chunks_per_seg(seg_len)) * 16, 256);
+}
+
+cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                         uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
+                         cudaStream_t stream);
+
+// ---------------------------------------------------------------- generator
+constexpr uint32_t kGenStatChunk = 65536;   // elements per statistics work item
+constexpr int kGenThreads = 256;
+constexpr uint32_t kMaxShards = 1024;
+constexpr uint32_t kMaxOutliers = 256;
+
+struct GenLayout {
+  size_t outlier_mask, flip_mask, stage_sigma, seg_coef, stats, total;
+  uint32_t mask_words;          // ceil(d / 32)
+  uint64_t stat_chunks;         // per segment
+};
+GenLayout gen_layout(const cg_pipeline_desc &d);
+
+struct GenParams {
+  uint64_t seed;
+  uint32_t S, N, T, d;
+  uint64_t L;                   // T * d
+  uint32_t config_id;
+  int32_t noise, tamper;
+  float sigma, lognormal, outlier_scale, tamper_param;
+  uint32_t n_outlier, n_flip;   // flipped channels per malicious stage
+  uint32_t mask_words;
+  uint64_t stat_chunks;
+  uint32_t mal_bits[kMaxShards / 32];
+};
+
+cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int8_t *labels,
+                            void *ws, const GenLayout &lay, int32_t *status, cudaStream_t stream);
+
+cudaError_t launch_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                uint32_t first, uint32_t n, uint32_t *out, cudaStream_t stream);
+cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                  uint32_t first, uint32_t n, float *out, cudaStream_t stream);
+
+// ---------------------------------------------------------------- ranking
+constexpr uint32_t kMaxRankShards = 1024;
+cudaError_t launch_control_labels(const int8_t *labels, uint32_t C, uint32_t N, uint32_t S,
+                                  uint64_t seed, uint32_t config_id0, int8_t *ctrl,
+                                  int32_t *status, cudaStream_t stream);
+cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, uint32_t N,
+                         uint32_t S, int64_t *u2, int64_t *gt, int64_t *eq, double *auroc,
+                         int32_t *status, cudaStream_t stream);
+
+}  // namespace cg

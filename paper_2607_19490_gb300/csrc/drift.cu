@@ -1,0 +1,231 @@
+// drift.cu -- the per-(stage, canary) drift reduction (Eq. 4 and the cosine
+// mismatch of the Sec. 4.4 ablation), the HBM-bound hot loop of the
+// verifier: every fp16 live element and every fp32 reference element is
+// read exactly once (6 bytes per element).
+//
+// Pass 1 (drift_partial_kernel): the [S][N][L] element space is cut into
+// work items of at most kDriftChunk elements, never crossing a segment.  A
+// persistent grid (SM count x resident blocks) walks the items in order.
+// Each thread streams 16-byte vectors (8 fp16 live values, 2 x 4 fp32
+// references) with non-allocating, 256-byte-prefetching global loads, four
+// vectors in flight, and accumulates in fp32:
+//     D = sum (h - a)^2,   E = sum (h - a)(h + a) = sum h^2 - a^2,
+//     A = sum a^2,         M = max |h - a|
+// The block reduces its sums with warp shuffles and a fixed tree and writes
+// one float4 per item.  Pass 2 (drift_finalize_kernel) combines the items of
+// a segment in order in fp64 and writes the three scores.  No atomics, so
+// the result is the same on every run.
+#include <cuda_fp16.h>
+
+#include "cg_internal.h"
+
+namespace cg {
+namespace {
+
+struct Acc {
+  float d, e, a, m;
+};
+
+__device__ __forceinline__ void acc_one(float h, float a, Acc &s) {
+  const float diff = h - a;
+  s.d = fmaf(diff, diff, s.d);
+  s.e = fmaf(diff, h + a, s.e);
+  s.a = fmaf(a, a, s.a);
+  s.m = fmaxf(s.m, fabsf(diff));
+}
+
+__device__ __forceinline__ uint4 ld_stream(const void *p) {
+  uint4 r;
+  asm("ld.global.nc.L1::no_allocate.L2::256B.v4.u32 {%0, %1, %2, %3}, [%4];"
+      : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+      : "l"(p));
+  return r;
+}
+
+__device__ __forceinline__ float2 half2_bits_to_float2(uint32_t bits) {
+  __half2 h;
+  memcpy(&h, &bits, 4);
+  return __half22float2(h);
+}
+
+// Eight elements: hv = 8 halves, r0/r1 = 8 floats.  A local sum of the
+// eight terms is added to the running sums (shorter fp32 chains).
+__device__ __forceinline__ void acc_eight(const uint4 hv, const uint4 r0, const uint4 r1, Acc &s) {
+  Acc t = {0.f, 0.f, 0.f, s.m};
+  float2 h;
+  h = half2_bits_to_float2(hv.x);
+  acc_one(h.x, __uint_as_float(r0.x), t);
+  acc_one(h.y, __uint_as_float(r0.y), t);
+  h = half2_bits_to_float2(hv.y);
+  acc_one(h.x, __uint_as_float(r0.z), t);
+  acc_one(h.y, __uint_as_float(r0.w), t);
+  h = half2_bits_to_float2(hv.z);
+  acc_one(h.x, __uint_as_float(r1.x), t);
+  acc_one(h.y, __uint_as_float(r1.y), t);
+  h = half2_bits_to_float2(hv.w);
+  acc_one(h.x, __uint_as_float(r1.z), t);
+  acc_one(h.y, __uint_as_float(r1.w), t);
+  s.d += t.d;
+  s.e += t.e;
+  s.a += t.a;
+  s.m = t.m;
+}
+
+__device__ __forceinline__ float half_bits_to_float(uint16_t b) {
+  return __half2float(__ushort_as_half(b));
+}
+
+constexpr int kUnroll = 4;
+
+__global__ void __launch_bounds__(kDriftThreads)
+drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ refs,
+                     uint64_t L, uint64_t chunks_per_seg, uint64_t n_items,
+                     float4 *__restrict__ partials) {
+  __shared__ Acc warp_acc[kDriftThreads / 32];
+  const int tid = threadIdx.x;
+  for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x) {
+    const uint64_t seg = item / chunks_per_seg;
+    const uint64_t ch = item - seg * chunks_per_seg;
+    const uint64_t seg0 = seg * L;
+    const uint64_t g0 = seg0 + ch * kDriftChunk;
+    const uint64_t g1 = min(g0 + (uint64_t)kDriftChunk, seg0 + L);
+    Acc s = {0.f, 0.f, 0.f, 0.f};
+
+    uint64_t v0 = (g0 + 7) & ~(uint64_t)7;
+    uint64_t v1 = g1 & ~(uint64_t)7;
+    if (v0 >= v1) {          // no aligned 8-vector inside: all scalar
+      v0 = g1;
+      v1 = g1;
+    }
+    // scalar head [g0, v0) and tail [v1, g1): fewer than 8 elements each,
+    // or the whole item when it has no aligned vector
+    for (uint64_t g = g0 + tid; g < v0; g += kDriftThreads)
+      acc_one(half_bits_to_float(acts[g]), refs[g], s);
+    for (uint64_t g = v1 + tid; g < g1; g += kDriftThreads)
+      acc_one(half_bits_to_float(acts[g]), refs[g], s);
+
+    const uint64_t nv = (v1 - v0) >> 3;
+    for (uint64_t i = tid; i < nv; i += (uint64_t)kUnroll * kDriftThreads) {
+      uint4 hv[kUnroll], r0[kUnroll], r1[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const uint64_t k = i + (uint64_t)u * kDriftThreads;
+        if (k < nv) {
+          const uint64_t g = v0 + 8 * k;
+          hv[u] = ld_stream(acts + g);
+          r0[u] = ld_stream(refs + g);
+          r1[u] = ld_stream(refs + g + 4);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        if (i + (uint64_t)u * kDriftThreads < nv) acc_eight(hv[u], r0[u], r1[u], s);
+      }
+    }
+
+    // block reduction: shuffle tree inside each warp, then warp 0 in order
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      s.d += __shfl_down_sync(0xFFFFFFFFu, s.d, off);
+      s.e += __shfl_down_sync(0xFFFFFFFFu, s.e, off);
+      s.a += __shfl_down_sync(0xFFFFFFFFu, s.a, off);
+      s.m = fmaxf(s.m, __shfl_down_sync(0xFFFFFFFFu, s.m, off));
+    }
+    if ((tid & 31) == 0) warp_acc[tid >> 5] = s;
+    __syncthreads();
+    if (tid < 32) {
+      Acc t = (tid < kDriftThreads / 32) ? warp_acc[tid] : Acc{0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+      for (int off = 4; off > 0; off >>= 1) {
+        t.d += __shfl_down_sync(0xFFFFFFFFu, t.d, off);
+        t.e += __shfl_down_sync(0xFFFFFFFFu, t.e, off);
+        t.a += __shfl_down_sync(0xFFFFFFFFu, t.a, off);
+        t.m = fmaxf(t.m, __shfl_down_sync(0xFFFFFFFFu, t.m, off));
+      }
+      if (tid == 0) partials[item] = make_float4(t.d, t.e, t.a, t.m);
+    }
+    __syncthreads();   // warp_acc is reused by the next item
+  }
+}
+
+// Scores of one segment from its fp64 sums.
+//   rel_l2  = sqrt(D / A)                                  (Eq. 4)
+//   cos_dev = 1 - h.a / (|h| |a|) with H = A + E, evaluated as
+//             (D - E^2 / (sqrt H + sqrt A)^2) / (2 sqrt(H A)), which equals
+//             (D - (sqrt H - sqrt A)^2) / (2 sqrt(H A)) without cancelling
+//             two near-equal norms.
+__global__ void drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg,
+                                      uint32_t S, uint32_t N, float *__restrict__ scores,
+                                      uint64_t stat_stride) {
+  const uint64_t seg = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (seg >= (uint64_t)S * N) return;
+  double D = 0.0, E = 0.0, A = 0.0;
+  float M = 0.f;
+  const float4 *p = partials + seg * chunks_per_seg;
+  for (uint64_t c = 0; c < chunks_per_seg; ++c) {
+    const float4 v = p[c];
+    D += (double)v.x;
+    E += (double)v.y;
+    A += (double)v.z;
+    M = fmaxf(M, v.w);
+  }
+  double rel, cosd;
+  if (isnan(D) || isnan(A)) {
+    rel = NAN;
+  } else if (A > 0.0) {
+    rel = sqrt(D / A);
+  } else {
+    rel = (D == 0.0) ? 0.0 : INFINITY;
+  }
+  const double H = A + E;
+  if (isnan(D) || isnan(E) || isnan(A)) {
+    cosd = NAN;
+  } else if (H > 0.0 && A > 0.0) {
+    const double sh = sqrt(H), sa = sqrt(A);
+    const double gap = E / (sh + sa);
+    cosd = (D - gap * gap) / (2.0 * sh * sa);
+    cosd = fmin(fmax(cosd, 0.0), 2.0);
+  } else {
+    cosd = 0.0;
+  }
+  const uint32_t s = (uint32_t)(seg / N), n = (uint32_t)(seg % N);
+  const uint64_t o = (uint64_t)n * S + s;
+  scores[o] = (float)rel;
+  scores[stat_stride + o] = M;
+  scores[2 * stat_stride + o] = (float)cosd;
+}
+
+}  // namespace
+
+cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                         uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
+                         cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  const uint64_t n_seg = (uint64_t)S * N;
+  const uint64_t cps = drift_chunks_per_seg(seg_len);
+  const uint64_t n_items = n_seg * cps;
+  float4 *partials = reinterpret_cast<float4 *>(static_cast<char *>(ws) + kDriftHeader);
+  uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
+  if (grid > n_items) grid = n_items;
+  if (grid < 1) grid = 1;
+  drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
+                                                                     n_items, partials);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  const unsigned fin_threads = 128;
+  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
+  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
+                                                                          scores, stat_stride);
+  return cudaGetLastError();
+}
+
+int drift_occupancy() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, drift_partial_kernel, kDriftThreads, 0) !=
+      cudaSuccess)
+    return 0;
+  return n;
+}
+
+}  // namespace cg

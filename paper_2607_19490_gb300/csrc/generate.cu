@@ -1,0 +1,392 @@
+// generate.cu -- device-side synthetic pipeline (Eq. 1-3 stand-in, Sec. 3.3).
+//
+// Materialises, for one configuration, the fp32 hop references and the fp16
+// live activations of every (stage, canary) segment, plus the labels:
+//   gen_setup_kernel    per-configuration draws: outlier-channel mask,
+//                       per-stage sigma (lognormal spread), flipped-channel
+//                       masks of the malicious stages; labels [N][S]
+//   gen_stats_kernel    per-segment sums the live values depend on:
+//                       sum |a| (Eq. 2: mu = ||a||_1 / (T d)) for benign
+//                       stages under the Eq. 2 noise model; sum a^2 and
+//                       sum g^2 (the Gaussian tamper's ||v|| and ||g||)
+//   gen_coef_kernel     per-segment scalar from those sums (fixed order, fp64)
+//   gen_materialise_kernel  per 8 elements: Philox normals, reference,
+//                       benign noise or tamper, 16-byte stores
+// Random draws follow the counter layout of cg_rng.cuh: element e of
+// segment seg on stream k uses block e / 4 of counter
+// (e / 4, seg, 4 config_id + k, 0).
+#include <cuda_fp16.h>
+
+#include "cg_internal.h"
+#include "cg_rng.cuh"
+
+namespace cg {
+namespace {
+
+__device__ __forceinline__ bool mask_bit(const uint32_t *mask, uint32_t c) {
+  return (__ldg(mask + (c >> 5)) >> (c & 31)) & 1u;
+}
+
+__device__ __forceinline__ bool is_malicious(const GenParams &p, uint32_t s) {
+  return (p.mal_bits[s >> 5] >> (s & 31)) & 1u;
+}
+
+// ----------------------------------------------------------------- setup
+// One block.  Threads first clear the masks; then thread 0 draws the
+// outlier channels, one thread per stage draws its sigma, and one thread per
+// malicious stage draws its flipped channels (each writes only its own mask
+// row).  Distinct values come from successive bounded draws with duplicates
+// redrawn; the draw count is capped and a cap hit is reported.
+__global__ void gen_setup_kernel(GenParams p, uint32_t *outlier_mask, uint32_t *flip_mask,
+                                 float *stage_sigma, int8_t *labels, int32_t *status) {
+  const int tid = threadIdx.x;
+  for (uint32_t i = tid; i < p.mask_words; i += blockDim.x) outlier_mask[i] = 0u;
+  for (uint64_t i = tid; i < (uint64_t)p.S * p.mask_words; i += blockDim.x) flip_mask[i] = 0u;
+  __syncthreads();
+  bool gave_up = false;
+  if (tid == 0 && p.n_outlier > 0) {
+    AuxWords w = aux_words(p.seed, kAuxOutlier, 0, p.config_id);
+    uint32_t got = 0;
+    const uint64_t cap = 64ull * p.d + 1024;
+    for (uint64_t tries = 0; got < p.n_outlier; ++tries) {
+      if (tries >= cap) { gave_up = true; break; }
+      const uint32_t c = aux_bounded(w, p.d, &gave_up);
+      const uint32_t bit = 1u << (c & 31);
+      if (outlier_mask[c >> 5] & bit) continue;
+      outlier_mask[c >> 5] |= bit;
+      ++got;
+    }
+  }
+  for (uint32_t s = tid; s < p.S; s += blockDim.x) {
+    float sig = p.sigma;
+    if (p.lognormal > 0.f) {
+      AuxWords w = aux_words(p.seed, kAuxStageSigma, s, p.config_id);
+      const uint32_t x0 = aux_next(w), x1 = aux_next(w);
+      sig = p.sigma * expf(p.lognormal * box_muller(x0, x1).x);
+    }
+    stage_sigma[s] = sig;
+    if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS && is_malicious(p, s)) {
+      uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
+      AuxWords w = aux_words(p.seed, kAuxFlip, s, p.config_id);
+      uint32_t got = 0;
+      const uint64_t cap = 64ull * p.d + 1024;
+      for (uint64_t tries = 0; got < p.n_flip; ++tries) {
+        if (tries >= cap) { gave_up = true; break; }
+        const uint32_t c = aux_bounded(w, p.d, &gave_up);
+        const uint32_t bit = 1u << (c & 31);
+        if (row[c >> 5] & bit) continue;
+        row[c >> 5] |= bit;
+        ++got;
+      }
+    }
+  }
+  if (labels) {
+    for (uint64_t i = tid; i < (uint64_t)p.N * p.S; i += blockDim.x)
+      labels[i] = is_malicious(p, (uint32_t)(i % p.S)) ? 1 : 0;
+  }
+  if (gave_up && status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
+}
+
+// Reference value of element e (segment-local) whose normal is z.
+__device__ __forceinline__ float ref_value(float z, uint32_t c, const GenParams &p,
+                                           const uint32_t *outlier_mask) {
+  if (p.n_outlier > 0 && mask_bit(outlier_mask, c)) return z * p.outlier_scale;
+  return z;
+}
+
+// ----------------------------------------------------------------- stats
+// Work item = (segment, chunk of kGenStatChunk elements).  Benign stages
+// under the Eq. 2 model sum |a|; malicious stages under the Gaussian tamper
+// sum a^2 and g^2.  Other segments write zeros.  One double2 per item.
+__global__ void __launch_bounds__(kGenThreads)
+gen_stats_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
+                 double2 *__restrict__ stats) {
+  __shared__ double2 warp_sum[kGenThreads / 32];
+  const uint64_t n_items = (uint64_t)p.S * p.N * p.stat_chunks;
+  const uint2 key = philox_key(p.seed);
+  const int tid = threadIdx.x;
+  for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x) {
+    const uint32_t seg = (uint32_t)(item / p.stat_chunks);
+    const uint64_t ch = item - (uint64_t)seg * p.stat_chunks;
+    const uint32_t s = seg / p.N;
+    const bool mal = is_malicious(p, s);
+    const bool need_l1 = !mal && p.noise == CG_NOISE_PAPER;
+    const bool need_l2 = mal && p.tamper == CG_TAMPER_ADDITIVE;
+    float x = 0.f, y = 0.f;
+    if (need_l1 || need_l2) {
+      const uint64_t e_begin = ch * kGenStatChunk;
+      const uint64_t e_end = min(e_begin + (uint64_t)kGenStatChunk, p.L);
+      // blocks of 4 elements; e_begin is a multiple of 4
+      for (uint64_t q = (e_begin >> 2) + tid; 4 * q < e_end; q += kGenThreads) {
+        const float4 z = normals4(key, (uint32_t)q, seg, 4u * p.config_id + kStreamRef);
+        const float zz[4] = {z.x, z.y, z.z, z.w};
+        float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (need_l2) g = normals4(key, (uint32_t)q, seg, 4u * p.config_id + kStreamTamper);
+        const float gg[4] = {g.x, g.y, g.z, g.w};
+        uint32_t c = (uint32_t)((4 * q) % p.d);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          if (4 * q + j < e_end) {
+            const float a = ref_value(zz[j], c, p, outlier_mask);
+            if (need_l1) {
+              x += fabsf(a);
+            } else {
+              x = fmaf(a, a, x);
+              y = fmaf(gg[j], gg[j], y);
+            }
+          }
+          c = (c + 1 == p.d) ? 0 : c + 1;
+        }
+      }
+    }
+    double dx = x, dy = y;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      dx += __shfl_down_sync(0xFFFFFFFFu, dx, off);
+      dy += __shfl_down_sync(0xFFFFFFFFu, dy, off);
+    }
+    if ((tid & 31) == 0) warp_sum[tid >> 5] = make_double2(dx, dy);
+    __syncthreads();
+    if (tid == 0) {
+      double2 t = make_double2(0.0, 0.0);
+      for (int w = 0; w < kGenThreads / 32; ++w) {
+        t.x += warp_sum[w].x;
+        t.y += warp_sum[w].y;
+      }
+      stats[item] = t;
+    }
+    __syncthreads();
+  }
+}
+
+// ----------------------------------------------------------------- coef
+// Per segment: benign MULT -> sigma_s; benign PAPER -> sigma_s * mu with
+// mu = sum|a| / L (Eq. 2); malicious ADDITIVE -> eps sqrt(sum a^2 / sum g^2)
+// (tau(v) = v + eps ||v|| g / ||g||); SCALE -> beta; otherwise 0.
+__global__ void gen_coef_kernel(GenParams p, const double2 *__restrict__ stats,
+                                const float *__restrict__ stage_sigma, float *__restrict__ coef) {
+  const uint64_t seg = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (seg >= (uint64_t)p.S * p.N) return;
+  const uint32_t s = (uint32_t)(seg / p.N);
+  double x = 0.0, y = 0.0;
+  const double2 *st = stats + seg * p.stat_chunks;
+  for (uint64_t c = 0; c < p.stat_chunks; ++c) {
+    x += st[c].x;
+    y += st[c].y;
+  }
+  float v = 0.f;
+  if (!is_malicious(p, s)) {
+    v = (p.noise == CG_NOISE_PAPER) ? (float)((double)stage_sigma[s] * (x / (double)p.L))
+                                    : stage_sigma[s];
+  } else if (p.tamper == CG_TAMPER_ADDITIVE) {
+    v = (y > 0.0) ? (float)((double)p.tamper_param * sqrt(x) / sqrt(y)) : 0.f;
+  } else if (p.tamper == CG_TAMPER_SCALE) {
+    v = p.tamper_param;
+  }
+  coef[seg] = v;
+}
+
+// ----------------------------------------------------------------- materialise
+// One thread per group of 8 segment-local elements (two Philox blocks per
+// stream).  Vector stores when the group is whole and 8-aligned globally.
+__global__ void __launch_bounds__(kGenThreads)
+gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
+                       const uint32_t *__restrict__ flip_mask, const float *__restrict__ coef,
+                       uint16_t *__restrict__ acts, float *__restrict__ refs) {
+  const uint64_t groups_per_seg = (p.L + 7) >> 3;
+  const uint64_t total = (uint64_t)p.S * p.N * groups_per_seg;
+  const uint2 key = philox_key(p.seed);
+  const uint32_t c2_ref = 4u * p.config_id + kStreamRef;
+  const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
+  const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
+  for (uint64_t gi = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < total;
+       gi += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t seg = (uint32_t)(gi / groups_per_seg);
+    const uint64_t j = gi - (uint64_t)seg * groups_per_seg;
+    const uint32_t s = seg / p.N;
+    const uint64_t e0 = 8 * j;
+    const int cnt = (int)min((uint64_t)8, p.L - e0);
+    const uint32_t q0 = (uint32_t)(2 * j);
+
+    float z[8], a[8], h[8];
+    {
+      const float4 z0 = normals4(key, q0, seg, c2_ref);
+      z[0] = z0.x; z[1] = z0.y; z[2] = z0.z; z[3] = z0.w;
+      if (cnt > 4) {
+        const float4 z1 = normals4(key, q0 + 1, seg, c2_ref);
+        z[4] = z1.x; z[5] = z1.y; z[6] = z1.z; z[7] = z1.w;
+      } else {
+        z[4] = z[5] = z[6] = z[7] = 0.f;
+      }
+    }
+    const uint32_t c0 = (uint32_t)(e0 % p.d);
+    uint32_t chan[8];
+    {
+      uint32_t c = c0;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        chan[k] = c;
+        c = (c + 1 == p.d) ? 0 : c + 1;
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a[k] = ref_value(z[k], chan[k], p, outlier_mask);
+
+    const bool mal = is_malicious(p, s);
+    const float cf = coef[seg];
+    if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
+      const uint32_t c2 = mal ? c2_tamper : c2_noise;
+      float n[8];
+      const float4 n0 = normals4(key, q0, seg, c2);
+      n[0] = n0.x; n[1] = n0.y; n[2] = n0.z; n[3] = n0.w;
+      if (cnt > 4) {
+        const float4 n1 = normals4(key, q0 + 1, seg, c2);
+        n[4] = n1.x; n[5] = n1.y; n[6] = n1.z; n[7] = n1.w;
+      } else {
+        n[4] = n[5] = n[6] = n[7] = 0.f;
+      }
+      if (!mal && p.noise == CG_NOISE_MULT) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[k] = a[k] * (1.0f + cf * n[k]);   // a (1 + sigma_s z)
+      } else {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[k] = fmaf(cf, n[k], a[k]);        // a + coef z
+      }
+    } else if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS) {
+      const uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = mask_bit(row, chan[k]) ? -a[k] : a[k];
+    } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = -a[k];
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = cf * a[k];
+    }
+
+    const uint64_t g = (uint64_t)seg * p.L + e0;
+    if (cnt == 8 && (g & 7) == 0) {
+      float4 *r4 = reinterpret_cast<float4 *>(refs + g);
+      r4[0] = make_float4(a[0], a[1], a[2], a[3]);
+      r4[1] = make_float4(a[4], a[5], a[6], a[7]);
+      uint4 hv;
+      hv.x = (uint32_t)__half_as_ushort(__float2half_rn(h[0])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[1])) << 16);
+      hv.y = (uint32_t)__half_as_ushort(__float2half_rn(h[2])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[3])) << 16);
+      hv.z = (uint32_t)__half_as_ushort(__float2half_rn(h[4])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[5])) << 16);
+      hv.w = (uint32_t)__half_as_ushort(__float2half_rn(h[6])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[7])) << 16);
+      *reinterpret_cast<uint4 *>(acts + g) = hv;
+    } else {
+      for (int k = 0; k < cnt; ++k) {
+        refs[g + k] = a[k];
+        acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
+      }
+    }
+  }
+}
+
+// ----------------------------------------------------------------- test views
+__global__ void philox_words_kernel(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                    uint32_t first, uint32_t n, uint4 *out) {
+  const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  out[i] = philox4x32_10(make_uint4(first + i, c1, c2, c3), philox_key(seed));
+}
+
+__global__ void philox_normals_kernel(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                      uint32_t first, uint32_t n, float4 *out) {
+  const uint32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint4 w = philox4x32_10(make_uint4(first + i, c1, c2, c3), philox_key(seed));
+  const float2 a = box_muller(w.x, w.y), b = box_muller(w.z, w.w);
+  out[i] = make_float4(a.x, a.y, b.x, b.y);
+}
+
+}  // namespace
+
+GenLayout gen_layout(const cg_pipeline_desc &d) {
+  GenLayout g;
+  const uint64_t L = (uint64_t)d.tokens * d.hidden;
+  g.mask_words = (d.hidden + 31) / 32;
+  g.stat_chunks = (L + kGenStatChunk - 1) / kGenStatChunk;
+  const uint64_t n_seg = (uint64_t)d.n_shards * d.n_canaries;
+  size_t off = 256;   // reserved
+  g.outlier_mask = off;
+  off = align_up(off + (size_t)g.mask_words * 4, 256);
+  g.flip_mask = off;
+  off = align_up(off + (size_t)d.n_shards * g.mask_words * 4, 256);
+  g.stage_sigma = off;
+  off = align_up(off + (size_t)d.n_shards * 4, 256);
+  g.seg_coef = off;
+  off = align_up(off + (size_t)n_seg * 4, 256);
+  g.stats = off;
+  off = align_up(off + (size_t)(n_seg * g.stat_chunks) * 16, 256);
+  g.total = off;
+  return g;
+}
+
+cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int8_t *labels,
+                            void *ws, const GenLayout &lay, int32_t *status, cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  char *base = static_cast<char *>(ws);
+  uint32_t *outlier_mask = reinterpret_cast<uint32_t *>(base + lay.outlier_mask);
+  uint32_t *flip_mask = reinterpret_cast<uint32_t *>(base + lay.flip_mask);
+  float *stage_sigma = reinterpret_cast<float *>(base + lay.stage_sigma);
+  float *coef = reinterpret_cast<float *>(base + lay.seg_coef);
+  double2 *stats = reinterpret_cast<double2 *>(base + lay.stats);
+
+  cudaError_t err;
+  gen_setup_kernel<<<1, 256, 0, stream>>>(p, outlier_mask, flip_mask, stage_sigma, labels, status);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+
+  const uint64_t n_seg = (uint64_t)p.S * p.N;
+  const bool any_stats = (p.noise == CG_NOISE_PAPER) || (p.tamper == CG_TAMPER_ADDITIVE);
+  const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)info.gen_blocks_per_sm;
+  if (any_stats) {
+    const uint64_t n_items = n_seg * p.stat_chunks;
+    const uint64_t grid = n_items < resident ? n_items : resident;
+    gen_stats_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, outlier_mask, stats);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  } else {
+    if ((err = cudaMemsetAsync(stats, 0, (size_t)n_seg * p.stat_chunks * 16, stream)) !=
+        cudaSuccess)
+      return err;
+  }
+  gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, stats, stage_sigma, coef);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+
+  const uint64_t groups = n_seg * ((p.L + 7) >> 3);
+  const uint64_t blocks_needed = (groups + kGenThreads - 1) / kGenThreads;
+  const uint64_t grid = blocks_needed < resident * 4 ? blocks_needed : resident * 4;
+  gen_materialise_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, outlier_mask, flip_mask,
+                                                                     coef, acts, refs);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                uint32_t first, uint32_t n, uint32_t *out, cudaStream_t stream) {
+  philox_words_kernel<<<(n + 255) / 256, 256, 0, stream>>>(seed, c1, c2, c3, first, n,
+                                                           reinterpret_cast<uint4 *>(out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
+                                  uint32_t first, uint32_t n, float *out, cudaStream_t stream) {
+  philox_normals_kernel<<<(n + 255) / 256, 256, 0, stream>>>(seed, c1, c2, c3, first, n,
+                                                             reinterpret_cast<float4 *>(out));
+  return cudaGetLastError();
+}
+
+int gen_occupancy() {
+  int n = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_materialise_kernel, kGenThreads, 0) !=
+      cudaSuccess)
+    return 0;
+  return n;
+}
+
+}  // namespace cg

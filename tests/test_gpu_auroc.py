@@ -1,0 +1,93 @@
+"""GPU parity of the ranking test: Mann-Whitney counts (bit-exact), A-hat
+(bit-exact) and the scrambled-label control labels (bit-exact) against the
+oracle on the same seeded inputs."""
+import numpy as np
+import pytest
+
+import seeded_inputs as SI
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def cg():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_19490_gb300 as m
+    m.build()
+    return m
+
+
+def run(cg, scores, labels, status=None):
+    import torch
+    res = cg.cg_auroc(torch.from_numpy(scores).cuda(), torch.from_numpy(labels).cuda(),
+                      status=status)
+    return {k: (v.cpu().numpy() if v is not None else None) for k, v in res.items()}
+
+
+@pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
+    (1, 1, 2, 1, 0, None), (5, 7, 4, 1, 0, None), (3, 64, 16, 1, 0, 3), (4, 9, 32, 3, 2, 5),
+    (2, 5, 33, 2, 0, 4), (2, 3, 100, 7, 5, None), (1, 2, 1024, 10, 3, 6), (324, 64, 16, 1, 0, None),
+    (6, 300, 8, 2, 1, 2),
+])
+def test_auroc_matches_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
+    scores, labels = SI.score_arrays(C, N, S, seed=C + N + S, n_malicious=n_mal,
+                                     tie_levels=ties, excluded=excluded)
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    for k in ("u2", "gt", "eq"):
+        assert np.array_equal(g[k], o[k]), k
+    assert np.array_equal(g["auroc"].view(np.uint64), o["auroc"].view(np.uint64))
+
+
+def test_auroc_nonuniform_pairs_bit_exact(cg, orc):
+    scores, labels = SI.score_arrays(3, 40, 9, seed=4, n_malicious=2, tie_levels=5)
+    labels[:, ::3, 8] = -1
+    labels[1, 5, :] = 0
+    labels[2, :, :] = 0           # no pair anywhere: A-hat is NaN
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    assert np.array_equal(g["u2"], o["u2"])
+    assert np.array_equal(g["auroc"][:2].view(np.uint64), o["auroc"][:2].view(np.uint64))
+    assert np.isnan(g["auroc"][2]) and np.isnan(o["auroc"][2])
+
+
+def test_auroc_stress_batch(cg, orc):
+    """65,536 configurations x 64 canaries x 16 stages."""
+    rng = np.random.Generator(np.random.PCG64(5))
+    C, N, S = 65536, 64, 16
+    scores = rng.random((C, N, S), dtype=np.float32)
+    labels = np.zeros((C, N, S), np.int8)
+    labels[np.arange(C), :, rng.integers(0, S, size=C)] = 1
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    assert np.array_equal(g["u2"], o["u2"])
+    assert np.array_equal(g["auroc"].view(np.uint64), o["auroc"].view(np.uint64))
+
+
+def test_auroc_nan_flag(cg):
+    import torch
+    scores, labels = SI.score_arrays(2, 3, 4, seed=1)
+    scores[1, 2, 0] = np.nan
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    run(cg, scores, labels, status=st)
+    status, word = cg.cg_read_status(st)
+    assert status == 4 and word & cg.DEVFLAG_NAN_SCORE
+
+
+@pytest.mark.parametrize("C,N,S,n_mal", [(1, 50, 4, 1), (3, 64, 16, 2), (2, 7, 33, 5), (4, 9, 1000, 3)])
+def test_control_labels_bit_exact(cg, orc, C, N, S, n_mal):
+    import torch
+    _, labels = SI.score_arrays(C, N, S, seed=S, n_malicious=n_mal, excluded=1)
+    ctrl = cg.cg_make_control_labels(torch.from_numpy(labels).cuda(), seed=77, config_id0=9)
+    assert np.array_equal(ctrl.cpu().numpy(), orc.control_labels(labels, seed=77, config_id0=9))
+
+
+def test_control_no_benign_flag(cg):
+    import torch
+    labels = np.ones((1, 2, 3), np.int8)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    cg.cg_make_control_labels(torch.from_numpy(labels).cuda(), seed=1, status=st)
+    status, word = cg.cg_read_status(st)
+    assert status == 8 and word == cg.DEVFLAG_NO_BENIGN

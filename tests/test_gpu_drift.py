@@ -1,0 +1,127 @@
+"""GPU parity of the drift reduction (Eq. 4, cosine ablation, max-abs) against
+the fp64 oracle on the same bytes.  Inputs come from seeded_inputs (numpy),
+never from the CUDA path.  Shapes span several work items (16384 elements
+each), ragged tails and segment starts that are not 16-byte aligned."""
+import numpy as np
+import pytest
+
+import seeded_inputs as SI
+from tests._cmp import assert_scores_close
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def cg():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_19490_gb300 as m
+    m.build()
+    return m
+
+
+def run(cg, acts, refs, S, N, **kw):
+    import torch
+    d_acts = torch.from_numpy(acts.view(np.float16)).cuda()
+    d_refs = torch.from_numpy(refs).cuda()
+    return cg.cg_drift_scores(d_acts, d_refs, S, N, **kw)
+
+
+@pytest.mark.parametrize("S,N,L", [
+    (2, 3, 1), (2, 3, 7), (2, 3, 8), (3, 2, 9), (4, 4, 100), (2, 2, 16384), (2, 3, 16385),
+    (3, 5, 40003), (1, 2, 65536 + 5), (5, 7, 4096), (4, 16, 8192),
+])
+def test_drift_matches_oracle(cg, orc, S, N, L):
+    acts, refs = SI.drift_arrays(S, N, L, seed=S * 1000 + N * 10 + L)
+    g = run(cg, acts, refs, S, N).cpu().numpy()
+    o = orc.drift_scores(acts, refs, S, N)
+    assert_scores_close(g, o, what=f"S={S} N={N} L={L}")
+
+
+def test_drift_paper_regimes(cg, orc):
+    """Benign floor, Gaussian tamper, sign flip, rescale: the regimes of Sec. 3.2."""
+    S, N, L = 4, 6, 3000
+    rels = np.array([1e-3, 5e-2, 2.0, 1e-4])[:, None, None] * np.ones((S, N, 1))
+    acts, refs = SI.drift_arrays(S, N, L, seed=77, rel=rels)
+    g = run(cg, acts, refs, S, N).cpu().numpy()
+    assert_scores_close(g, orc.drift_scores(acts, refs, S, N))
+
+
+def test_drift_oracle_generated_bytes(cg, orc):
+    """The oracle's own synthetic pipeline bytes (tiny workload and a rescale)."""
+    for cfg in (SI.TINY, SI.shrink(SI.TINY, tamper=SI.TAMPER_SCALE, tamper_param=1.05)):
+        o_acts, o_refs, _ = orc.generate_pipeline(orc.desc_from_dict(cfg))
+        S, N = cfg["n_shards"], cfg["n_canaries"]
+        g = run(cg, o_acts, o_refs, S, N).cpu().numpy()
+        assert_scores_close(g, orc.drift_scores(o_acts, o_refs, S, N))
+
+
+def test_drift_stat_stride_and_sentinels(cg, orc):
+    import torch
+    S, N, L = 3, 4, 1000
+    acts, refs = SI.drift_arrays(S, N, L, seed=3)
+    C, c = 5, 2                                  # place this config at slot 2 of 5
+    big = torch.full((3, C, N, S), -7.0, dtype=torch.float32, device="cuda")
+    view = big.view(-1)[c * N * S:]
+    run(cg, acts, refs, S, N, scores=view, stat_stride=C * N * S)
+    out = big.cpu().numpy()
+    o = orc.drift_scores(acts, refs, S, N)
+    assert_scores_close(out[:, c], o)
+    mask = np.ones(C, bool)
+    mask[c] = False
+    assert np.all(out[:, mask] == -7.0)
+
+
+def test_drift_nan_and_edge_values(cg, orc):
+    S, N, L = 2, 2, 33
+    acts, refs = SI.drift_arrays(S, N, L, seed=9)
+    a = acts.view(np.float16).copy()
+    a[1, 1, 5] = np.nan
+    g = run(cg, a.view(np.uint16), refs, S, N).cpu().numpy()
+    o = orc.drift_scores(a.view(np.uint16), refs, S, N)
+    assert_scores_close(g, o)
+    assert np.isnan(g[0, 1, 1]) and np.isnan(g[2, 1, 1]) and np.isfinite(g[1, 1, 1])
+
+
+def test_drift_deterministic(cg):
+    S, N, L = 4, 8, 50000
+    acts, refs = SI.drift_arrays(S, N, L, seed=1)
+    g1 = run(cg, acts, refs, S, N).cpu().numpy()
+    g2 = run(cg, acts, refs, S, N).cpu().numpy()
+    assert np.array_equal(g1.view(np.uint32), g2.view(np.uint32))
+
+
+def test_drift_full_size_planted_segments(cg, orc):
+    """70B-like workload at full size in the benchmark's launch configuration:
+    neutral host bytes are planted into sampled segments of the generated
+    pipeline, and those segments' scores are compared with the oracle."""
+    import torch
+    cfg = SI.SEVENTY_B
+    S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
+    desc = cg.PipelineDesc.from_config(cfg)
+    acts, refs, labels = cg.cg_generate_pipeline(desc)
+    picks = [(0, 0), (7, 13), (15, 255), (3, 128)]
+    planted = {}
+    for i, (s, n) in enumerate(picks):
+        pa, pr = SI.drift_arrays(1, 1, L, seed=500 + i)
+        acts[s, n].copy_(torch.from_numpy(pa.view(np.float16).reshape(-1)))
+        refs[s, n].copy_(torch.from_numpy(pr.reshape(-1)))
+        planted[(s, n)] = (pa.reshape(-1), pr.reshape(-1))
+    ws = torch.empty(cg.cg_drift_workspace_size(S, N, L), dtype=torch.uint8, device="cuda")
+    scores = cg.cg_drift_scores(acts, refs, S, N, ws=ws).cpu().numpy()
+    for (s, n), (pa, pr) in planted.items():
+        out, _ = orc.drift_segment(pa, pr)
+        assert_scores_close(scores[:, n, s][:, None], out[:, None], what=f"segment {(s, n)}")
+    # properties of every generated segment: benign floor O(sigma) (Sec. 3.4),
+    # channel-flip tamper far above it, and the full detector separates them
+    mal = cfg["malicious"][0]
+    keep = np.ones((N, S), bool)
+    for s, n in picks:
+        keep[n, s] = False
+    rel = scores[0]
+    benign = rel[:, [s for s in range(S) if s != mal]][keep[:, [s for s in range(S) if s != mal]]]
+    assert np.all((benign > 0.3 * cfg["benign_sigma"]) & (benign < 3 * cfg["benign_sigma"]))
+    assert np.all(rel[keep[:, mal], mal] > 0.1)
+    del acts, refs
+    torch.cuda.empty_cache()
