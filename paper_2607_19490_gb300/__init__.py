@@ -155,6 +155,8 @@ def cg_philox_words(seed, c1, c2, c3, first_block, n_blocks, out=None, stream=No
     if out is None:
         out = torch.empty((n_blocks, 4), dtype=torch.int32, device="cuda")
     _cuda(out, "out", (torch.int32,))
+    if out.numel() < 4 * n_blocks:
+        raise ValueError("out must hold 4 * n_blocks words")
     _check(load().cg_philox_words(seed, c1, c2, c3, first_block, n_blocks, _ptr(out),
                                   _stream(stream)), "cg_philox_words")
     return out
@@ -165,6 +167,8 @@ def cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, out=None, stream=
     if out is None:
         out = torch.empty((n_blocks, 4), dtype=torch.float32, device="cuda")
     _cuda(out, "out", (torch.float32,))
+    if out.numel() < 4 * n_blocks:
+        raise ValueError("out must hold 4 * n_blocks floats")
     _check(load().cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, _ptr(out),
                                     _stream(stream)), "cg_philox_normals")
     return out
@@ -235,6 +239,10 @@ def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=N
     _cuda(scores, "scores", (torch.float32,))
     _cuda(ws, "ws", (torch.uint8,))
     _cuda(status, "status", (torch.int32,))
+    if scores.numel() < 2 * stat_stride + n_seg:
+        raise ValueError("scores must hold 2 * stat_stride + N * S floats")
+    if ws.numel() < cg_drift_workspace_size(n_shards, n_canaries, seg_len):
+        raise ValueError("workspace smaller than cg_drift_workspace_size")
     _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
                                   _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
                                   _stream(stream)), "cg_drift_scores")
