@@ -173,6 +173,36 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
                           int32_t *d_status, cg_stream_t stream);
 
 /*
+ * cg_drift_scores without a workspace: same arguments, layouts and results
+ * as cg_drift_scores, but the per-chunk partial sums go to a fixed 4 MiB
+ * array of device memory inside the library, so the call allocates nothing
+ * and needs no scratch buffer from the caller.  The paper has no
+ * counterpart; this exists for callers that cannot allocate device memory
+ * on their scoring path: a verifier embedded in an inference server whose
+ * memory pool already holds nearly all of HBM (weights and KV cache) and
+ * gives plug-ins no allocator, or a serving loop that cannot afford the
+ * device-wide synchronisation cudaMalloc/cudaFree may cause.
+ *   Limit: n_shards * n_canaries * ceil(seg_len / CG_NOALLOC_CHUNK_ELEMENTS)
+ *   <= CG_NOALLOC_MAX_WORK_ITEMS (e.g. 4096 segments of 2^20 elements);
+ *   larger problems return CG_ERR_UNSUPPORTED before any launch.
+ *   The array is loaded on every GPU that loads the library and held until
+ *   the process exits.  The first call on each device looks up the array's
+ *   device address (cudaGetSymbolAddress) with that device current; make
+ *   that first call before any stream capture.
+ *   Every call shares the array: calls that overlap on the GPU (on
+ *   different streams or from different host threads) race and corrupt
+ *   each other's results; serialise them on one stream.  Nothing in it
+ *   needs to start at zero: every partial is written before it is read.
+ */
+#define CG_NOALLOC_CHUNK_ELEMENTS 16384u
+#define CG_NOALLOC_MAX_WORK_ITEMS 262144u
+cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,
+                                  uint32_t n_shards, uint32_t n_canaries,
+                                  uint64_t seg_len, float *d_scores,
+                                  uint64_t stat_stride, int32_t *d_status,
+                                  cg_stream_t stream);
+
+/*
  * Scrambled-label negative control (Sec. 4.5).  For every configuration c
  * and canary n, a stage j* is drawn uniformly from the stages labelled 0 in
  * d_labels (ascending order; Philox aux stream 4 with config id

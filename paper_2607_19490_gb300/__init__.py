@@ -20,6 +20,7 @@ __all__ = [
     "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
     "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
+    "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
     "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
@@ -94,6 +95,7 @@ def load() -> ctypes.CDLL:
             "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
+            "cg_drift_scores_noalloc": ([P, P, u32, u32, u64, P, u64, P, P], ctypes.c_int),
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
             "cg_auroc": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
             "cg_read_status": ([P, P, ctypes.POINTER(i32)], ctypes.c_int),
@@ -246,6 +248,34 @@ def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=N
     _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
                                   _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
                                   _stream(stream)), "cg_drift_scores")
+    return scores
+
+
+def cg_drift_scores_noalloc(acts, refs, n_shards, n_canaries, scores, stat_stride=None,
+                            status=None, stream=None):
+    """cg_drift_scores without a workspace, for callers that cannot allocate
+    device memory while scoring (for example a verifier living inside an
+    inference server whose memory pool owns nearly all of HBM).  The library
+    keeps the partial sums in a fixed 4 MiB device array shared by every
+    call, so calls must not overlap on the GPU; problems above
+    CG_NOALLOC_MAX_WORK_ITEMS chunks of 16384 elements are rejected.  The
+    caller passes the output buffer; nothing is allocated here."""
+    torch = _torch()
+    _cuda(acts, "acts", (torch.float16,))
+    _cuda(refs, "refs", (torch.float32,))
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(status, "status", (torch.int32,))
+    n_seg = n_shards * n_canaries
+    if acts.numel() != refs.numel() or acts.numel() % n_seg:
+        raise ValueError("acts and refs must both hold S*N*L elements")
+    seg_len = acts.numel() // n_seg
+    if stat_stride is None:
+        stat_stride = n_seg
+    if scores.numel() < 2 * stat_stride + n_seg:
+        raise ValueError("scores must hold 2 * stat_stride + N * S floats")
+    _check(load().cg_drift_scores_noalloc(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
+                                          _ptr(scores), stat_stride, _ptr(status),
+                                          _stream(stream)), "cg_drift_scores_noalloc")
     return scores
 
 

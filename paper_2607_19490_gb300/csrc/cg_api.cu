@@ -7,6 +7,10 @@
 
 #include "cg_internal.h"
 
+static_assert(CG_NOALLOC_MAX_WORK_ITEMS == cg::kNoallocDriftItems,
+              "public limit and scratch size disagree");
+static_assert(CG_NOALLOC_CHUNK_ELEMENTS == cg::kDriftChunk, "public chunk and kernel chunk disagree");
+
 namespace cg {
 
 int drift_occupancy();
@@ -186,6 +190,25 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs, uint32_t 
   (void)d_status;   // the streaming path has no device-side failure mode
   return from_cuda(cg::launch_drift(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores,
                                     stat_stride, d_ws, (cudaStream_t)stream));
+}
+
+cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,
+                                  uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
+                                  float *d_scores, uint64_t stat_stride, int32_t *d_status,
+                                  cg_stream_t stream) {
+  if (n_shards == 0 || n_canaries == 0 || seg_len == 0) return CG_ERR_INVALID_ARG;
+  const uint64_t n_seg = (uint64_t)n_shards * n_canaries;
+  if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
+  if (n_seg * cg::drift_chunks_per_seg(seg_len) > CG_NOALLOC_MAX_WORK_ITEMS)
+    return CG_ERR_UNSUPPORTED;
+  if (!d_acts || !d_refs || !d_scores) return CG_ERR_INVALID_ARG;
+  if (stat_stride < n_seg) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || !aligned(d_scores, 4) ||
+      (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  (void)d_status;
+  return from_cuda(cg::launch_drift_noalloc(d_acts, d_refs, n_shards, n_canaries, seg_len,
+                                            d_scores, stat_stride, (cudaStream_t)stream));
 }
 
 cg_status cg_make_control_labels(const int8_t *d_labels, uint32_t n_configs,

@@ -39,6 +39,12 @@ cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, ui
                          uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
                          cudaStream_t stream);
 
+// Work-item capacity of the fixed scratch array used by cg_drift_scores_noalloc.
+constexpr uint64_t kNoallocDriftItems = 262144;
+cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                                 uint64_t seg_len, float *scores, uint64_t stat_stride,
+                                 cudaStream_t stream);
+
 // ---------------------------------------------------------------- generator
 constexpr uint32_t kGenStatChunk = 65536;   // elements per statistics work item
 constexpr int kGenThreads = 256;

@@ -17,6 +17,8 @@
 // the result is the same on every run.
 #include <cuda_fp16.h>
 
+#include <mutex>
+
 #include "cg_internal.h"
 
 namespace cg {
@@ -226,6 +228,65 @@ int drift_occupancy() {
       cudaSuccess)
     return 0;
   return n;
+}
+
+}  // namespace cg
+
+// ----------------------------------------------------------------- no-alloc variant
+// Scratch for cg_drift_scores_noalloc: the per-item partial sums live in a
+// fixed device array owned by the library instead of a caller workspace.
+// 262,144 float4 items = 4 MiB, held on every GPU that loads the library
+// until the process exits.  All calls share it, so calls that overlap on the
+// GPU (different streams, or other host threads) race on it.
+static __device__ __align__(256) float4 g_drift_scratch[cg::kNoallocDriftItems];
+
+namespace cg {
+namespace {
+std::mutex g_scratch_mu;
+float4 *g_scratch_ptr[64] = {};
+}  // namespace
+
+// Device address of g_drift_scratch on the current device, looked up once
+// per device (cudaGetSymbolAddress; the host-side symbol is only a stand-in).
+static cudaError_t noalloc_scratch(float4 **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_ptr[dev]) {
+    void *p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_drift_scratch);
+    if (e != cudaSuccess) return e;
+    g_scratch_ptr[dev] = static_cast<float4 *>(p);
+  }
+  *out = g_scratch_ptr[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                                 uint64_t seg_len, float *scores, uint64_t stat_stride,
+                                 cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  float4 *partials = nullptr;
+  cudaError_t err = noalloc_scratch(&partials);
+  if (err != cudaSuccess) return err;
+  const uint64_t n_seg = (uint64_t)S * N;
+  const uint64_t cps = drift_chunks_per_seg(seg_len);
+  const uint64_t n_items = n_seg * cps;
+  uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
+  if (grid > n_items) grid = n_items;
+  if (grid < 1) grid = 1;
+  drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
+                                                                     n_items, partials);
+  err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  const unsigned fin_threads = 128;
+  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
+  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
+                                                                          scores, stat_stride);
+  return cudaGetLastError();
 }
 
 }  // namespace cg
