@@ -173,6 +173,22 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
                           int32_t *d_status, cg_stream_t stream);
 
 /*
+ * cg_drift_scores with the live activations in pinned host memory: the
+ * drift kernel reads h_acts directly over the host-GPU link (one pass, no
+ * staging copy in HBM) while the references stay resident in device memory,
+ * as the verifier's stored fp32 references do (Sec. 3.3).  h_acts must be
+ * page-locked host memory known to CUDA (cudaHostAlloc or cudaHostRegister);
+ * anything else returns CG_ERR_INVALID_ARG before any launch.  It must stay
+ * unmodified until the call's work on `stream` completes.  All other
+ * arguments, layouts and results are those of cg_drift_scores.
+ */
+cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs,
+                               uint32_t n_shards, uint32_t n_canaries,
+                               uint64_t seg_len, float *d_scores,
+                               uint64_t stat_stride, void *d_ws, size_t ws_bytes,
+                               int32_t *d_status, cg_stream_t stream);
+
+/*
  * cg_drift_scores without a workspace: same arguments, layouts and results
  * as cg_drift_scores, but the per-chunk partial sums go to a fixed 4 MiB
  * array of device memory inside the library, so the call allocates nothing

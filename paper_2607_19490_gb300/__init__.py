@@ -20,7 +20,7 @@ __all__ = [
     "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
     "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
-    "cg_drift_scores_noalloc",
+    "cg_drift_scores_host", "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
     "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
@@ -95,6 +95,7 @@ def load() -> ctypes.CDLL:
             "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
+            "cg_drift_scores_host": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_noalloc": ([P, P, u32, u32, u64, P, u64, P, P], ctypes.c_int),
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
             "cg_auroc": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
@@ -248,6 +249,42 @@ def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=N
     _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
                                   _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
                                   _stream(stream)), "cg_drift_scores")
+    return scores
+
+
+def cg_drift_scores_host(h_acts, refs, n_shards, n_canaries, scores=None, stat_stride=None,
+                         ws=None, status=None, stream=None):
+    """Drift scores with the live activations in pinned host memory (a CPU
+    fp16 tensor with pin_memory=True); the kernel reads them directly over
+    the host link and the fp32 references stay on the device."""
+    torch = _torch()
+    if h_acts.is_cuda or not h_acts.is_pinned():
+        raise ValueError("h_acts must be a pinned CPU tensor")
+    if not h_acts.is_contiguous() or h_acts.dtype != torch.float16:
+        raise ValueError("h_acts must be contiguous float16")
+    _cuda(refs, "refs", (torch.float32,))
+    n_seg = n_shards * n_canaries
+    if h_acts.numel() != refs.numel() or h_acts.numel() % n_seg:
+        raise ValueError("h_acts and refs must both hold S*N*L elements")
+    seg_len = h_acts.numel() // n_seg
+    if scores is None:
+        scores = torch.empty((3, n_canaries, n_shards), dtype=torch.float32, device=refs.device)
+        stat_stride = n_seg
+    if stat_stride is None:
+        stat_stride = n_seg
+    if ws is None:
+        ws = torch.empty(cg_drift_workspace_size(n_shards, n_canaries, seg_len), dtype=torch.uint8,
+                         device=refs.device)
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    if scores.numel() < 2 * stat_stride + n_seg:
+        raise ValueError("scores must hold 2 * stat_stride + N * S floats")
+    if ws.numel() < cg_drift_workspace_size(n_shards, n_canaries, seg_len):
+        raise ValueError("workspace smaller than cg_drift_workspace_size")
+    _check(load().cg_drift_scores_host(_ptr(h_acts), _ptr(refs), n_shards, n_canaries, seg_len,
+                                       _ptr(scores), stat_stride, _ptr(ws), ws.numel(),
+                                       _ptr(status), _stream(stream)), "cg_drift_scores_host")
     return scores
 
 

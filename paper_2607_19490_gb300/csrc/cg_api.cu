@@ -192,6 +192,25 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs, uint32_t 
                                     stat_stride, d_ws, (cudaStream_t)stream));
 }
 
+cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs, uint32_t n_shards,
+                               uint32_t n_canaries, uint64_t seg_len, float *d_scores,
+                               uint64_t stat_stride, void *d_ws, size_t ws_bytes,
+                               int32_t *d_status, cg_stream_t stream) {
+  if (!h_acts) return CG_ERR_INVALID_ARG;
+  // Only page-locked host memory registered with CUDA may be read by a
+  // kernel; resolve its device-side address (equal to the host address
+  // under unified addressing).
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, h_acts) != cudaSuccess) {
+    cudaGetLastError();
+    return CG_ERR_INVALID_ARG;
+  }
+  if (attr.type != cudaMemoryTypeHost || attr.devicePointer == nullptr) return CG_ERR_INVALID_ARG;
+  return cg_drift_scores(static_cast<const uint16_t *>(attr.devicePointer), d_refs, n_shards,
+                         n_canaries, seg_len, d_scores, stat_stride, d_ws, ws_bytes, d_status,
+                         stream);
+}
+
 cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,
                                   uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
                                   float *d_scores, uint64_t stat_stride, int32_t *d_status,

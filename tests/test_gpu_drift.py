@@ -125,3 +125,27 @@ def test_drift_full_size_planted_segments(cg, orc):
     assert np.all(rel[keep[:, mal], mal] > 0.1)
     del acts, refs
     torch.cuda.empty_cache()
+
+
+def test_drift_host_live_activations(cg, orc):
+    """Live activations read from pinned host memory give the same scores as
+    from device memory (same kernel, same order) and match the oracle."""
+    import torch
+    S, N, L = 3, 5, 40003
+    acts, refs = SI.drift_arrays(S, N, L, seed=21)
+    h_acts = torch.from_numpy(acts.view(np.float16)).pin_memory()
+    d_refs = torch.from_numpy(refs).cuda()
+    g_host = cg.cg_drift_scores_host(h_acts, d_refs, S, N).cpu().numpy()
+    g_dev = cg.cg_drift_scores(h_acts.cuda(), d_refs, S, N).cpu().numpy()
+    assert np.array_equal(g_host.view(np.uint32), g_dev.view(np.uint32))
+    assert_scores_close(g_host, orc.drift_scores(acts, refs, S, N))
+
+
+def test_drift_host_rejects_pageable(cg):
+    import ctypes
+    L = cg.load()
+    buf = (ctypes.c_uint16 * 64)()          # ordinary (pageable) host memory
+    fake = ctypes.c_void_p(0x10000)
+    st = L.cg_drift_scores_host(ctypes.cast(buf, ctypes.c_void_p), fake, 2, 2, 16, fake, 4, fake,
+                                1 << 20, None, None)
+    assert st == 1
