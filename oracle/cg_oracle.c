@@ -50,11 +50,14 @@ enum { OR_TAMPER_ADDITIVE = 0, OR_TAMPER_SIGNFLIP_CHANNELS = 1,
 /*                     4 * config_id + stream, 0)                           */
 /*   auxiliary words: (word index / 4, (purpose << 24) | sub,               */
 /*                     4 * config_id + OR_STREAM_AUX, 0)                    */
-/* so config_id must stay below 2^30 and c3 is always 0.                    */
+/* so config_id must stay below 2^30.  c3 is 0 for every draw of the live   */
+/* pipeline; an independent benign recompute r (the redundant-recompute      */
+/* ceiling and the noisy-reference ablation, Sec. 4.4-4.5) draws its noise   */
+/* with c3 = r, so replica 0 is the live draw itself.                        */
 enum { OR_STREAM_REF = 0, OR_STREAM_NOISE = 1, OR_STREAM_TAMPER = 2,
        OR_STREAM_AUX = 3 };
 enum { OR_AUX_OUTLIER = 1, OR_AUX_SHARD_SIGMA = 2, OR_AUX_FLIP = 3,
-       OR_AUX_CONTROL = 4 };
+       OR_AUX_CONTROL = 4, OR_AUX_RANDOM = 5 };
 
 /* ------------------------------------------------------------------------ */
 /* Philox4x32-10 (SC'11, Sec. 5): ten rounds of the two-multiply S-box with   */
@@ -354,15 +357,48 @@ int or_config_tables(const or_desc *D, uint32_t *outlier, double *shard_sigma,
 }
 
 /* The normal of element e of segment seg on stream `stream`.                */
-static double element_normal(const uint32_t key[2], uint32_t seg,
-                             uint32_t config_id, uint32_t stream, uint64_t e) {
-  uint32_t ctr[4] = {(uint32_t)(e >> 2), seg, 4u * config_id + stream, 0u};
+static double element_normal_r(const uint32_t key[2], uint32_t seg,
+                               uint32_t config_id, uint32_t stream, uint32_t c3,
+                               uint64_t e) {
+  uint32_t ctr[4] = {(uint32_t)(e >> 2), seg, 4u * config_id + stream, c3};
   uint32_t w[4];
   or_philox4x32_10(ctr, key, w);
   double z[4];
   or_box_muller(w[0], w[1], &z[0], &z[1]);
   or_box_muller(w[2], w[3], &z[2], &z[3]);
   return z[e & 3];
+}
+
+static double element_normal(const uint32_t key[2], uint32_t seg,
+                             uint32_t config_id, uint32_t stream, uint64_t e) {
+  return element_normal_r(key, seg, config_id, stream, 0u, e);
+}
+
+/* Benign output of stage s on segment (s, n) with the noise of replica r   */
+/* (Eq. 2): MULT a (1 + sigma_s z), PAPER a + sigma_s mu z.                  */
+static void benign_values(const or_desc *D, const or_tables *t, uint32_t s,
+                          uint32_t seg, const double *a, uint64_t L,
+                          uint32_t replica, double *live, double *coef_out) {
+  uint32_t key[2];
+  seed_to_key(D->seed, key);
+  double sig = t->shard_sigma[s];
+  double coef = 0.0;
+  if (D->noise == OR_NOISE_MULT) {
+    for (uint64_t e = 0; e < L; ++e) {
+      double z = element_normal_r(key, seg, D->config_id, OR_STREAM_NOISE, replica, e);
+      live[e] = a[e] * (1.0 + sig * z);
+    }
+  } else {
+    double l1 = 0.0;
+    for (uint64_t e = 0; e < L; ++e) l1 += fabs(a[e]);
+    double mu = l1 / (double)L;
+    coef = sig * mu;
+    for (uint64_t e = 0; e < L; ++e) {
+      double z = element_normal_r(key, seg, D->config_id, OR_STREAM_NOISE, replica, e);
+      live[e] = a[e] + coef * z;
+    }
+  }
+  if (coef_out) *coef_out = coef;
 }
 
 /* One (stage s, canary n) segment of T*d elements, token-major.             */
@@ -399,24 +435,7 @@ static int segment(const or_desc *D, const or_tables *t, uint32_t s,
 
   double coef = 0.0;
   if (!t->is_mal[s]) {
-    double sig = t->shard_sigma[s];
-    if (D->noise == OR_NOISE_MULT) {
-      /* relative per-element noise: h = a (1 + sigma z) */
-      for (uint64_t e = 0; e < L; ++e) {
-        double z = element_normal(key, seg, D->config_id, OR_STREAM_NOISE, e);
-        live[e] = a[e] * (1.0 + sig * z);
-      }
-    } else {
-      /* Eq. 2: delta ~ N(0, sigma^2 mu^2 I), mu = ||a||_1 / (T d) */
-      double l1 = 0.0;
-      for (uint64_t e = 0; e < L; ++e) l1 += fabs(a[e]);
-      double mu = l1 / (double)L;
-      coef = sig * mu;
-      for (uint64_t e = 0; e < L; ++e) {
-        double z = element_normal(key, seg, D->config_id, OR_STREAM_NOISE, e);
-        live[e] = a[e] + coef * z;
-      }
-    }
+    benign_values(D, t, s, seg, a, L, 0u, live, &coef);
   } else if (D->tamper == OR_TAMPER_ADDITIVE) {
     /* Gaussian tamper: tau(v) = v + eps ||v||_F g / ||g||_F */
     double aa = 0.0, gg = 0.0;
@@ -499,6 +518,73 @@ int or_generate_pipeline(const or_desc *D, uint16_t *acts, float *refs,
   free_tables(&t);
   (void)n_threads;
   return err;
+}
+
+/* An independent benign recompute of every stage (Sec. 4.5, redundant-     */
+/* recompute ceiling; Sec. 4.4, noisy reference): the benign output of each */
+/* stage, malicious ones included, with the noise of replica r, rounded to  */
+/* fp16 and stored as fp32 [S][N][T][d].  Replica 0 is the live draw.       */
+int or_generate_recompute(const or_desc *D, uint32_t replica, float *out,
+                          int n_threads) {
+  int st = check_desc(D);
+  if (st) return st;
+  or_tables t;
+  st = build_tables(D, &t);
+  if (st) return st;
+  const uint32_t S = D->n_shards, N = D->n_canaries, d = D->hidden;
+  const uint64_t L = (uint64_t)D->tokens * d;
+  int err = OR_OK;
+#ifdef _OPENMP
+  if (n_threads > 0) omp_set_num_threads(n_threads);
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+  for (int64_t q = 0; q < (int64_t)S * N; ++q) {
+    uint32_t s = (uint32_t)(q / N), n = (uint32_t)(q % N);
+    uint32_t seg = s * N + n;
+    uint32_t key[2];
+    seed_to_key(D->seed, key);
+    double *a = (double *)malloc(L * sizeof(double));
+    double *h = (double *)malloc(L * sizeof(double));
+    if (!a || !h) {
+      free(a); free(h);
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+      err = OR_NO_MEMORY;
+      continue;
+    }
+    for (uint64_t e = 0; e < L; ++e) {
+      uint32_t c = (uint32_t)(e % d);
+      double scale = 1.0;
+      for (uint32_t j = 0; j < D->n_outlier; ++j)
+        if (t.outlier[j] == c) scale = D->outlier_scale;
+      a[e] = (double)(float)(element_normal(key, seg, D->config_id,
+                                            OR_STREAM_REF, e) * scale);
+    }
+    benign_values(D, &t, s, seg, a, L, replica, h, NULL);
+    for (uint64_t e = 0; e < L; ++e)
+      out[(size_t)q * L + e] = (float)or_half_to_double(or_half_from_double(h[e]));
+    free(a);
+    free(h);
+  }
+  free_tables(&t);
+  (void)n_threads;
+  return err;
+}
+
+/* Random baseline (Sec. 4.5): every score replaced by Uniform(0, 1).        */
+/* scores[c][n][s] = (x >> 8) 2^-24, x = word s of aux stream (RANDOM, sub   */
+/* = canary n) with config id config_id0 + c.                                */
+void or_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C,
+                      uint32_t N, uint32_t S, float *out) {
+  for (uint32_t c = 0; c < C; ++c)
+    for (uint32_t n = 0; n < N; ++n) {
+      or_words w;
+      words_init(&w, seed, OR_AUX_RANDOM, n, config_id0 + c);
+      for (uint32_t s = 0; s < S; ++s)
+        out[((size_t)c * N + n) * S + s] =
+            (float)((double)(words_next(&w) >> 8) * 0x1p-24);
+    }
 }
 
 /* ------------------------------------------------------------------------ */

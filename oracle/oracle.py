@@ -30,7 +30,7 @@ OR_OK, OR_BAD_ARG, OR_NAN_SCORE, OR_NO_MEMORY = 0, 1, 2, 3
 NOISE_MULT, NOISE_PAPER = 0, 1
 TAMPER_ADDITIVE, TAMPER_SIGNFLIP_CHANNELS, TAMPER_SIGNFLIP_FULL, TAMPER_SCALE = 0, 1, 2, 3
 STREAM_REF, STREAM_NOISE, STREAM_TAMPER, STREAM_AUX = 0, 1, 2, 3
-AUX_OUTLIER, AUX_SHARD_SIGMA, AUX_FLIP, AUX_CONTROL = 1, 2, 3, 4
+AUX_OUTLIER, AUX_SHARD_SIGMA, AUX_FLIP, AUX_CONTROL, AUX_RANDOM = 1, 2, 3, 4, 5
 
 
 def build(force: bool = False) -> str:
@@ -104,6 +104,9 @@ def lib():
             L.or_control_labels.argtypes = [P(ctypes.c_int8), u32, u32, u32, u64, u32, P(ctypes.c_int8)]
             L.or_control_labels.restype = i32
             L.or_max_threads.restype = ctypes.c_int
+            L.or_generate_recompute.argtypes = [P(_Desc), u32, P(ctypes.c_float), ctypes.c_int]
+            L.or_generate_recompute.restype = i32
+            L.or_random_scores.argtypes = [u64, u32, u32, u32, u32, P(ctypes.c_float)]
         return _lib
 
 
@@ -222,6 +225,23 @@ def generate_pipeline(desc, n_threads=0):
                                       _p(refs, ctypes.c_float), _p(labels, ctypes.c_int8),
                                       int(n_threads)))
     return acts, refs, labels
+
+
+def generate_recompute(desc, replica, n_threads=0):
+    """Independent benign recompute of every stage: fp32 values of fp16
+    outputs [S][N][T*d] (the ceiling's and the noisy reference's comparator)."""
+    S, N, L = desc.n_shards, desc.n_canaries, desc.tokens * desc.hidden
+    out = np.zeros((S, N, L), dtype=np.float32)
+    _check(lib().or_generate_recompute(ctypes.byref(desc), replica, _p(out, ctypes.c_float),
+                                       int(n_threads)))
+    return out
+
+
+def random_scores(seed, C, N, S, config_id0=0):
+    """Random-baseline scores float32 [C][N][S], Uniform(0, 1)."""
+    out = np.zeros((C, N, S), dtype=np.float32)
+    lib().or_random_scores(seed, config_id0, C, N, S, _p(out, ctypes.c_float))
+    return out
 
 
 # --------------------------------------------------------------------------
