@@ -150,6 +150,30 @@ cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts,
                                size_t ws_bytes, int32_t *d_status,
                                cg_stream_t stream);
 
+/*
+ * An independent benign recompute of every stage, for the
+ * redundant-recompute ceiling (Sec. 4.5) and the noisy-reference ablation
+ * (Sec. 4.4): d_out (fp32 [S][N][T][d], 16-byte aligned) receives the fp16
+ * output of the benign computation of each stage -- malicious stages
+ * included, since the recompute is honest -- with its noise drawn from
+ * replica `replica` (Philox counter word 3).  Replica 0 reproduces the live
+ * benign draw of cg_generate_pipeline; passing d_out as the references of
+ * cg_drift_scores scores the live pipeline against the recompute.  The
+ * workspace is cg_generate_workspace_size(desc).
+ */
+cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica,
+                                float *d_out, void *d_ws, size_t ws_bytes,
+                                int32_t *d_status, cg_stream_t stream);
+
+/*
+ * Random-baseline scores (Sec. 4.5): d_scores[c][n][s] ~ Uniform(0, 1),
+ * the top 24 bits of word s of Philox aux stream 5 (canary n, config id
+ * config_id0 + c) times 2^-24.  fp32 [C][N][S], 4-byte aligned.
+ */
+cg_status cg_random_scores(uint64_t seed, uint32_t config_id0, uint32_t n_configs,
+                           uint32_t n_canaries, uint32_t n_shards, float *d_scores,
+                           cg_stream_t stream);
+
 /* Workspace bytes cg_drift_scores needs for S * N segments of seg_len. */
 cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
                                   uint64_t seg_len, size_t *bytes);
@@ -252,6 +276,22 @@ cg_status cg_auroc(const float *d_scores, const int8_t *d_labels,
                    uint32_t n_configs, uint32_t n_canaries, uint32_t n_shards,
                    int64_t *d_u2, int64_t *d_gt, int64_t *d_eq,
                    double *d_auroc, int32_t *d_status, cg_stream_t stream);
+
+/*
+ * Pooled Mann-Whitney AUROC: per configuration, every malicious score of
+ * every canary against every benign score of every canary (the U statistic
+ * the paper names as equivalent to its ranking test, Sec. 3.4; the
+ * per-canary mean of cg_auroc is Eq. 6 itself).  d_scores fp32 / d_labels
+ * int8 [C][N][S] as in cg_auroc.  Per configuration: d_u2[c] = 2 U (ties
+ * count one half), d_n_mal[c], d_n_ben[c] (may be NULL) and
+ * d_auroc[c] = u2 / (2 n_mal n_ben), one fp64 division of exact integers
+ * (NaN without a pair).  NaN scores are left out of the pool and raise
+ * CG_DEVFLAG_NAN_SCORE.  N * S up to 16384.
+ */
+cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels,
+                          uint32_t n_configs, uint32_t n_canaries, uint32_t n_shards,
+                          int64_t *d_u2, int64_t *d_n_mal, int64_t *d_n_ben,
+                          double *d_auroc, int32_t *d_status, cg_stream_t stream);
 
 /*
  * Synchronise `stream`, read the device status word and map it: 0 ->

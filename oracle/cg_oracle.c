@@ -729,6 +729,43 @@ int or_auroc(const float *scores, const int8_t *labels, uint32_t C,
   return status;
 }
 
+/* Pooled Mann-Whitney AUROC: all malicious scores of a configuration      */
+/* (every canary) against all its benign scores -- the U statistic the     */
+/* paper names as equivalent to its ranking test (Sec. 3.4).  Brute force   */
+/* over every (malicious, benign) pair of the configuration:               */
+/*   u2 = 2 #{m_i > m_j} + #{m_i = m_j},  A = u2 / (2 n_mal n_ben).          */
+/* NaN scores are left out of the pool and reported.                       */
+int or_auroc_pooled(const float *scores, const int8_t *labels, uint32_t C,
+                    uint32_t N, uint32_t S, int64_t *u2, int64_t *n_mal,
+                    int64_t *n_ben, double *auroc) {
+  int status = OR_OK;
+  const size_t per = (size_t)N * S;
+  for (uint32_t c = 0; c < C; ++c) {
+    const float *m = scores + (size_t)c * per;
+    const int8_t *l = labels + (size_t)c * per;
+    int64_t g = 0, e = 0, nm = 0, nb = 0;
+    for (size_t i = 0; i < per; ++i) {
+      if ((l[i] == 1 || l[i] == 0) && isnan(m[i])) { status = OR_NAN_SCORE; continue; }
+      if (l[i] == 1) nm++;
+      if (l[i] == 0) nb++;
+    }
+    for (size_t i = 0; i < per; ++i) {
+      if (l[i] != 1 || isnan(m[i])) continue;
+      for (size_t j = 0; j < per; ++j) {
+        if (l[j] != 0 || isnan(m[j])) continue;
+        if (m[i] > m[j]) g++;
+        else if (m[i] == m[j]) e++;
+      }
+    }
+    if (u2) u2[c] = 2 * g + e;
+    if (n_mal) n_mal[c] = nm;
+    if (n_ben) n_ben[c] = nb;
+    if (auroc)
+      auroc[c] = (nm * nb > 0) ? (double)(2 * g + e) / (double)(2 * nm * nb) : NAN;
+  }
+  return status;
+}
+
 /* ------------------------------------------------------------------------ */
 /* Scrambled-label negative control (Sec. 4.5): the true mismatches are kept */
 /* and, on every canary, a stage j* drawn uniformly from the benign stages   */

@@ -107,6 +107,10 @@ def lib():
             L.or_generate_recompute.argtypes = [P(_Desc), u32, P(ctypes.c_float), ctypes.c_int]
             L.or_generate_recompute.restype = i32
             L.or_random_scores.argtypes = [u64, u32, u32, u32, u32, P(ctypes.c_float)]
+            L.or_auroc_pooled.argtypes = [P(ctypes.c_float), P(ctypes.c_int8), u32, u32, u32,
+                                          P(ctypes.c_int64), P(ctypes.c_int64), P(ctypes.c_int64),
+                                          P(dbl)]
+            L.or_auroc_pooled.restype = i32
         return _lib
 
 
@@ -290,6 +294,26 @@ def auroc(scores, labels):
         raise OracleError("NaN score among labelled stages")
     _check(st)
     return {"u2": u2, "gt": gt, "eq": eq, "pairs": pairs, "auroc": A}
+
+
+def auroc_pooled(scores, labels, allow_nan=False):
+    """Pooled Mann-Whitney over all canaries of each configuration:
+    dict(u2, n_mal, n_ben, auroc) per configuration."""
+    sc = np.ascontiguousarray(scores, dtype=np.float32)
+    lb = np.ascontiguousarray(labels, dtype=np.int8)
+    C, N, S = sc.shape
+    u2 = np.zeros(C, np.int64)
+    nm = np.zeros(C, np.int64)
+    nb = np.zeros(C, np.int64)
+    A = np.zeros(C, np.float64)
+    st = lib().or_auroc_pooled(_p(sc, ctypes.c_float), _p(lb, ctypes.c_int8), C, N, S,
+                               _p(u2, ctypes.c_int64), _p(nm, ctypes.c_int64),
+                               _p(nb, ctypes.c_int64), _p(A, ctypes.c_double))
+    if st == OR_NAN_SCORE and not allow_nan:
+        raise OracleError("NaN score among labelled stages")
+    if st not in (OR_OK, OR_NAN_SCORE):
+        _check(st)
+    return {"u2": u2, "n_mal": nm, "n_ben": nb, "auroc": A}
 
 
 def control_labels(labels, seed, config_id0=0):

@@ -21,7 +21,8 @@ __all__ = [
     "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
     "cg_drift_scores_host", "cg_drift_scores_noalloc",
-    "cg_make_control_labels", "cg_auroc", "cg_read_status",
+    "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
+    "cg_random_scores", "cg_auroc_pooled",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
     "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
 ]
@@ -94,11 +95,14 @@ def load() -> ctypes.CDLL:
             "cg_generate_workspace_size": ([ctypes.POINTER(PipelineDesc), ctypes.POINTER(sz)], ctypes.c_int),
             "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
+            "cg_generate_recompute": ([ctypes.POINTER(PipelineDesc), u32, P, P, sz, P, P], ctypes.c_int),
+            "cg_random_scores": ([u64, u32, u32, u32, u32, P, P], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_host": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_noalloc": ([P, P, u32, u32, u64, P, u64, P, P], ctypes.c_int),
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
             "cg_auroc": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
+            "cg_auroc_pooled": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
             "cg_read_status": ([P, P, ctypes.POINTER(i32)], ctypes.c_int),
         }
         for name, (args, res) in sigs.items():
@@ -212,6 +216,40 @@ def cg_generate_pipeline(desc: PipelineDesc, acts=None, refs=None, labels=None, 
                                        _ptr(ws), ws.numel(), _ptr(status), _stream(stream)),
            "cg_generate_pipeline")
     return acts, refs, labels
+
+
+def cg_generate_recompute(desc: PipelineDesc, replica, out=None, ws=None, status=None,
+                          stream=None):
+    """Independent benign recompute of every stage as fp32 [S][N][T*d] (the
+    redundant-recompute ceiling's and the noisy reference's comparator)."""
+    torch = _torch()
+    S, N, L = desc.n_shards, desc.n_canaries, desc.seg_len
+    if out is None:
+        out = torch.empty((S, N, L), dtype=torch.float32, device="cuda")
+    if ws is None:
+        ws = torch.empty(cg_generate_workspace_size(desc), dtype=torch.uint8, device="cuda")
+    _cuda(out, "out", (torch.float32,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    if out.numel() != S * N * L:
+        raise ValueError("out must hold S*N*T*d elements")
+    _check(load().cg_generate_recompute(ctypes.byref(desc), replica, _ptr(out), _ptr(ws),
+                                        ws.numel(), _ptr(status), _stream(stream)),
+           "cg_generate_recompute")
+    return out
+
+
+def cg_random_scores(seed, n_configs, n_canaries, n_shards, config_id0=0, out=None, stream=None):
+    """Random-baseline scores fp32 [C][N][S] ~ Uniform(0, 1)."""
+    torch = _torch()
+    if out is None:
+        out = torch.empty((n_configs, n_canaries, n_shards), dtype=torch.float32, device="cuda")
+    _cuda(out, "out", (torch.float32,))
+    if out.numel() < n_configs * n_canaries * n_shards:
+        raise ValueError("out too small")
+    _check(load().cg_random_scores(seed, config_id0, n_configs, n_canaries, n_shards, _ptr(out),
+                                   _stream(stream)), "cg_random_scores")
+    return out
 
 
 def cg_drift_workspace_size(n_shards, n_canaries, seg_len) -> int:
@@ -357,6 +395,30 @@ def cg_auroc(scores, labels, u2=None, gt=None, eq=None, auroc=None, status=None,
     _check(load().cg_auroc(_ptr(scores), _ptr(labels), C, N, S, _ptr(u2), _ptr(gt), _ptr(eq),
                            _ptr(auroc), _ptr(status), _stream(stream)), "cg_auroc")
     return {"u2": u2, "gt": gt, "eq": eq, "auroc": auroc}
+
+
+def cg_auroc_pooled(scores, labels, u2=None, n_mal=None, n_ben=None, auroc=None, status=None,
+                    stream=None):
+    """Pooled Mann-Whitney AUROC per configuration of scores/labels [C][N][S]."""
+    torch = _torch()
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(labels, "labels", (torch.int8,))
+    if scores.shape != labels.shape or scores.dim() != 3:
+        raise ValueError("scores and labels must both be [C][N][S]")
+    C, N, S = scores.shape
+    dev = scores.device
+    u2 = torch.empty((C,), dtype=torch.int64, device=dev) if u2 is None else u2
+    n_mal = torch.empty((C,), dtype=torch.int64, device=dev) if n_mal is None else n_mal
+    n_ben = torch.empty((C,), dtype=torch.int64, device=dev) if n_ben is None else n_ben
+    auroc = torch.empty((C,), dtype=torch.float64, device=dev) if auroc is None else auroc
+    for t, n in ((u2, "u2"), (n_mal, "n_mal"), (n_ben, "n_ben")):
+        _cuda(t, n, (torch.int64,))
+    _cuda(auroc, "auroc", (torch.float64,))
+    _cuda(status, "status", (torch.int32,))
+    _check(load().cg_auroc_pooled(_ptr(scores), _ptr(labels), C, N, S, _ptr(u2), _ptr(n_mal),
+                                  _ptr(n_ben), _ptr(auroc), _ptr(status), _stream(stream)),
+           "cg_auroc_pooled")
+    return {"u2": u2, "n_mal": n_mal, "n_ben": n_ben, "auroc": auroc}
 
 
 def cg_read_status(status, stream=None):

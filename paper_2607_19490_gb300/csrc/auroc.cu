@@ -187,7 +187,146 @@ __global__ void control_labels_kernel(const int8_t *__restrict__ labels, uint32_
   }
 }
 
+// ----------------------------------------------------------------- pooled
+// Pooled Mann-Whitney over all canaries of a configuration.  One block per
+// configuration: the labelled scores become 64-bit keys
+// (order-preserving image of the float << 32 | label) in shared memory, a
+// bitonic network sorts them, and every malicious key adds twice its
+// midrank, lo + 1 + hi, where [lo, hi) is the run of its score found by
+// binary search.  2U = sum(2 midrank) - n_mal (n_mal + 1), exact in int64.
+constexpr int kPoolThreads = 1024;
+constexpr int kPoolWarps = kPoolThreads / 32;
+
+__device__ __forceinline__ uint32_t order_key(float x) {
+  uint32_t b = __float_as_uint(x);
+  if (b == 0x80000000u) b = 0u;                         // -0 ranks with +0
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+__device__ __forceinline__ uint32_t lower_bound_u64(const unsigned long long *k, uint32_t n,
+                                                    unsigned long long v) {
+  uint32_t lo = 0, hi = n;
+  while (lo < hi) {
+    const uint32_t mid = (lo + hi) >> 1;
+    if (k[mid] < v) lo = mid + 1;
+    else hi = mid;
+  }
+  return lo;
+}
+
+__global__ void __launch_bounds__(kPoolThreads)
+auroc_pooled_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                    uint32_t C, uint32_t per, uint32_t M, int64_t *__restrict__ u2_out,
+                    int64_t *__restrict__ nm_out, int64_t *__restrict__ nb_out,
+                    double *__restrict__ auroc, int32_t *status) {
+  extern __shared__ unsigned long long keys[];
+  __shared__ unsigned int count;
+  __shared__ long long red[kPoolWarps][3];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
+    if (tid == 0) count = 0u;
+    __syncthreads();
+    bool nan_seen = false;
+    const float *m = scores + (uint64_t)c * per;
+    const int8_t *l = labels + (uint64_t)c * per;
+    for (uint32_t i = tid; i < per; i += kPoolThreads) {
+      const int lab = l[i];
+      if (lab != 0 && lab != 1) continue;
+      const float x = m[i];
+      if (is_nan_f(x)) {
+        nan_seen = true;
+        continue;
+      }
+      const unsigned int pos = atomicAdd(&count, 1u);
+      keys[pos] = ((unsigned long long)order_key(x) << 32) | (unsigned long long)lab;
+    }
+    __syncthreads();
+    const uint32_t n = count;
+    for (uint32_t i = n + tid; i < M; i += kPoolThreads) keys[i] = ~0ull;   // pad: sorts last
+    __syncthreads();
+    for (uint32_t k = 2; k <= M; k <<= 1) {
+      for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+        for (uint32_t i = tid; i < M; i += kPoolThreads) {
+          const uint32_t ixj = i ^ j;
+          if (ixj > i) {
+            const unsigned long long a = keys[i], b = keys[ixj];
+            const bool up = (i & k) == 0;
+            if ((a > b) == up) {
+              keys[i] = b;
+              keys[ixj] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
+    }
+    long long rs = 0, nm = 0, nb = 0;
+    for (uint32_t i = tid; i < n; i += kPoolThreads) {
+      const unsigned long long v = keys[i];
+      if (v & 1ull) {
+        const unsigned long long hk = v >> 32;
+        const uint32_t lo = lower_bound_u64(keys, n, hk << 32);
+        const uint32_t hi = lower_bound_u64(keys, n, (hk + 1) << 32);
+        rs += (long long)lo + 1 + (long long)hi;
+        nm += 1;
+      } else {
+        nb += 1;
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      rs += __shfl_down_sync(0xFFFFFFFFu, rs, off);
+      nm += __shfl_down_sync(0xFFFFFFFFu, nm, off);
+      nb += __shfl_down_sync(0xFFFFFFFFu, nb, off);
+    }
+    if (lane == 0) {
+      red[warp][0] = rs;
+      red[warp][1] = nm;
+      red[warp][2] = nb;
+    }
+    if (__any_sync(0xFFFFFFFFu, nan_seen) && lane == 0 && status)
+      atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+    __syncthreads();
+    if (tid == 0) {
+      long long R = 0, NM = 0, NB = 0;
+      for (int w = 0; w < kPoolWarps; ++w) {
+        R += red[w][0];
+        NM += red[w][1];
+        NB += red[w][2];
+      }
+      const long long u2 = R - NM * (NM + 1);
+      u2_out[c] = u2;
+      if (nm_out) nm_out[c] = NM;
+      if (nb_out) nb_out[c] = NB;
+      auroc[c] = (NM * NB > 0) ? __ddiv_rn((double)u2, (double)(2 * NM * NB)) : NAN;
+    }
+    __syncthreads();
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint32_t C,
+                                uint32_t N, uint32_t S, int64_t *u2, int64_t *n_mal,
+                                int64_t *n_ben, double *auroc, int32_t *status,
+                                cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  const uint32_t per = N * S;
+  uint32_t M = 2;
+  while (M < per) M <<= 1;
+  const size_t smem = (size_t)M * sizeof(unsigned long long);
+  cudaError_t err = cudaFuncSetAttribute(auroc_pooled_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  uint64_t per_sm = smem > 0 ? (200u * 1024u) / (smem + 1024) : 1;
+  if (per_sm < 1) per_sm = 1;
+  uint64_t grid = (uint64_t)info.sm_count * per_sm;
+  if (grid > C) grid = C;
+  auroc_pooled_kernel<<<(unsigned)grid, kPoolThreads, smem, stream>>>(scores, labels, C, per, M, u2,
+                                                                      n_mal, n_ben, auroc, status);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, uint32_t N,
                          uint32_t S, int64_t *u2, int64_t *gt, int64_t *eq, double *auroc,

@@ -77,6 +77,36 @@ cg_status check_desc(const cg_pipeline_desc *d) {
   return CG_OK;
 }
 
+cg::GenParams make_params(const cg_pipeline_desc &d, const cg::GenLayout &lay) {
+  cg::GenParams p;
+  memset(&p, 0, sizeof(p));
+  p.seed = d.seed;
+  p.S = d.n_shards;
+  p.N = d.n_canaries;
+  p.T = d.tokens;
+  p.d = d.hidden;
+  p.L = (uint64_t)d.tokens * d.hidden;
+  p.config_id = d.config_id;
+  p.noise = d.noise;
+  p.tamper = d.tamper;
+  p.sigma = d.benign_sigma;
+  p.lognormal = d.shard_sigma_lognormal;
+  p.outlier_scale = d.outlier_scale;
+  p.tamper_param = d.tamper_param;
+  p.n_outlier = d.n_outlier;
+  // max(1, round-half-up(p d)) flipped channels, evaluated in double
+  double r = floor((double)d.tamper_param * (double)d.hidden + 0.5);
+  uint32_t nf = r < 1.0 ? 1u : (r > (double)d.hidden ? d.hidden : (uint32_t)r);
+  p.n_flip = nf;
+  p.mask_words = lay.mask_words;
+  p.stat_chunks = lay.stat_chunks;
+  for (uint32_t i = 0; i < d.n_malicious; ++i) {
+    const uint32_t s = (uint32_t)d.malicious[i];
+    p.mal_bits[s >> 5] |= 1u << (s & 31);
+  }
+  return p;
+}
+
 }  // namespace
 
 extern "C" {
@@ -136,34 +166,39 @@ cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts, f
   if (!d_ws || ws_bytes < lay.total) return CG_ERR_WORKSPACE;
   if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
 
-  cg::GenParams p;
-  memset(&p, 0, sizeof(p));
-  p.seed = desc->seed;
-  p.S = desc->n_shards;
-  p.N = desc->n_canaries;
-  p.T = desc->tokens;
-  p.d = desc->hidden;
-  p.L = (uint64_t)desc->tokens * desc->hidden;
-  p.config_id = desc->config_id;
-  p.noise = desc->noise;
-  p.tamper = desc->tamper;
-  p.sigma = desc->benign_sigma;
-  p.lognormal = desc->shard_sigma_lognormal;
-  p.outlier_scale = desc->outlier_scale;
-  p.tamper_param = desc->tamper_param;
-  p.n_outlier = desc->n_outlier;
-  // max(1, round-half-up(p d)) flipped channels, evaluated in double
-  double r = floor((double)desc->tamper_param * (double)desc->hidden + 0.5);
-  uint32_t nf = r < 1.0 ? 1u : (r > (double)desc->hidden ? desc->hidden : (uint32_t)r);
-  p.n_flip = nf;
-  p.mask_words = lay.mask_words;
-  p.stat_chunks = lay.stat_chunks;
-  for (uint32_t i = 0; i < desc->n_malicious; ++i) {
-    const uint32_t s = (uint32_t)desc->malicious[i];
-    p.mal_bits[s >> 5] |= 1u << (s & 31);
-  }
+  cg::GenParams p = make_params(*desc, lay);
   return from_cuda(cg::launch_generate(p, d_acts, d_refs, d_labels, d_ws, lay, d_status,
                                        (cudaStream_t)stream));
+}
+
+cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica, float *d_out,
+                                void *d_ws, size_t ws_bytes, int32_t *d_status,
+                                cg_stream_t stream) {
+  cg_status st = check_desc(desc);
+  if (st != CG_OK) return st;
+  if (!d_out) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_out, 16) || (d_status && !aligned(d_status, 4))) return CG_ERR_ALIGNMENT;
+  const cg::GenLayout lay = cg::gen_layout(*desc);
+  if (!d_ws || ws_bytes < lay.total) return CG_ERR_WORKSPACE;
+  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
+  cg::GenParams p = make_params(*desc, lay);
+  memset(p.mal_bits, 0, sizeof(p.mal_bits));   // the recompute is honest on every stage
+  p.recompute = 1;
+  p.noise_c3 = replica;
+  return from_cuda(cg::launch_generate(p, nullptr, d_out, nullptr, d_ws, lay, d_status,
+                                       (cudaStream_t)stream));
+}
+
+cg_status cg_random_scores(uint64_t seed, uint32_t config_id0, uint32_t n_configs,
+                           uint32_t n_canaries, uint32_t n_shards, float *d_scores,
+                           cg_stream_t stream) {
+  if (!d_scores || n_configs == 0 || n_canaries == 0 || n_shards == 0) return CG_ERR_INVALID_ARG;
+  if ((uint64_t)config_id0 + n_configs > (1ull << 30)) return CG_ERR_INVALID_ARG;
+  if (n_canaries > (1u << 24)) return CG_ERR_UNSUPPORTED;
+  if ((uint64_t)n_configs * n_canaries * n_shards >= (1ull << 40)) return CG_ERR_UNSUPPORTED;
+  if (!aligned(d_scores, 4)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_random_scores(seed, config_id0, n_configs, n_canaries, n_shards,
+                                            d_scores, (cudaStream_t)stream));
 }
 
 cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
@@ -259,6 +294,24 @@ cg_status cg_auroc(const float *d_scores, const int8_t *d_labels, uint32_t n_con
     return CG_ERR_ALIGNMENT;
   return from_cuda(cg::launch_auroc(d_scores, d_labels, n_configs, n_canaries, n_shards, d_u2,
                                     d_gt, d_eq, d_auroc, d_status, (cudaStream_t)stream));
+}
+
+cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels, uint32_t n_configs,
+                          uint32_t n_canaries, uint32_t n_shards, int64_t *d_u2,
+                          int64_t *d_n_mal, int64_t *d_n_ben, double *d_auroc, int32_t *d_status,
+                          cg_stream_t stream) {
+  if (!d_scores || !d_labels || !d_u2 || !d_auroc || n_configs == 0 || n_canaries == 0 ||
+      n_shards == 0)
+    return CG_ERR_INVALID_ARG;
+  if ((uint64_t)n_canaries * n_shards > cg::kMaxPooled) return CG_ERR_UNSUPPORTED;
+  if ((uint64_t)n_configs * n_canaries * n_shards >= (1ull << 40)) return CG_ERR_UNSUPPORTED;
+  if (!aligned(d_scores, 4) || !aligned(d_u2, 8) || !aligned(d_auroc, 8) ||
+      (d_n_mal && !aligned(d_n_mal, 8)) || (d_n_ben && !aligned(d_n_ben, 8)) ||
+      (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_auroc_pooled(d_scores, d_labels, n_configs, n_canaries, n_shards,
+                                           d_u2, d_n_mal, d_n_ben, d_auroc, d_status,
+                                           (cudaStream_t)stream));
 }
 
 cg_status cg_read_status(const int32_t *d_status, cg_stream_t stream, int32_t *h_word) {

@@ -68,11 +68,16 @@ struct GenParams {
   uint32_t n_outlier, n_flip;   // flipped channels per malicious stage
   uint32_t mask_words;
   uint64_t stat_chunks;
+  int32_t recompute;            // 1: write a benign recompute of every stage into refs
+  uint32_t noise_c3;            // counter word 3 of the noise stream (recompute replica)
   uint32_t mal_bits[kMaxShards / 32];
 };
 
 cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int8_t *labels,
                             void *ws, const GenLayout &lay, int32_t *status, cudaStream_t stream);
+
+cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
+                                 uint32_t S, float *out, cudaStream_t stream);
 
 cudaError_t launch_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
                                 uint32_t first, uint32_t n, uint32_t *out, cudaStream_t stream);
@@ -84,6 +89,11 @@ constexpr uint32_t kMaxRankShards = 1024;
 cudaError_t launch_control_labels(const int8_t *labels, uint32_t C, uint32_t N, uint32_t S,
                                   uint64_t seed, uint32_t config_id0, int8_t *ctrl,
                                   int32_t *status, cudaStream_t stream);
+constexpr uint32_t kMaxPooled = 16384;   // labelled scores per configuration (128 KiB of keys)
+cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint32_t C,
+                                uint32_t N, uint32_t S, int64_t *u2, int64_t *n_mal,
+                                int64_t *n_ben, double *auroc, int32_t *status,
+                                cudaStream_t stream);
 cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, uint32_t N,
                          uint32_t S, int64_t *u2, int64_t *gt, int64_t *eq, double *auroc,
                          int32_t *status, cudaStream_t stream);

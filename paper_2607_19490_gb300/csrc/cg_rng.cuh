@@ -21,7 +21,8 @@ constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
 // Stream ids folded into counter word 2 as 4 * config_id + stream.
 constexpr uint32_t kStreamRef = 0, kStreamNoise = 1, kStreamTamper = 2, kStreamAux = 3;
 // Purposes of auxiliary word streams (counter word 1 = purpose << 24 | sub).
-constexpr uint32_t kAuxOutlier = 1, kAuxStageSigma = 2, kAuxFlip = 3, kAuxControl = 4;
+constexpr uint32_t kAuxOutlier = 1, kAuxStageSigma = 2, kAuxFlip = 3, kAuxControl = 4,
+                   kAuxRandom = 5;
 
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
 #pragma unroll
@@ -51,9 +52,11 @@ __device__ __forceinline__ float2 box_muller(uint32_t x0, uint32_t x1) {
   return make_float2(r * c, r * s);
 }
 
-// The four normals of one Philox block.
-__device__ __forceinline__ float4 normals4(uint2 key, uint32_t q, uint32_t c1, uint32_t c2) {
-  const uint4 w = philox4x32_10(make_uint4(q, c1, c2, 0u), key);
+// The four normals of one Philox block (counter word 3 = c3: 0 for every
+// live draw, the replica index for an independent benign recompute).
+__device__ __forceinline__ float4 normals4(uint2 key, uint32_t q, uint32_t c1, uint32_t c2,
+                                           uint32_t c3 = 0u) {
+  const uint4 w = philox4x32_10(make_uint4(q, c1, c2, c3), key);
   const float2 a = box_muller(w.x, w.y);
   const float2 b = box_muller(w.z, w.w);
   return make_float4(a.x, a.y, b.x, b.y);

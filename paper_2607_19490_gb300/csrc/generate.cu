@@ -236,11 +236,12 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
     const float cf = coef[seg];
     if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
       const uint32_t c2 = mal ? c2_tamper : c2_noise;
+      const uint32_t c3 = mal ? 0u : p.noise_c3;
       float n[8];
-      const float4 n0 = normals4(key, q0, seg, c2);
+      const float4 n0 = normals4(key, q0, seg, c2, c3);
       n[0] = n0.x; n[1] = n0.y; n[2] = n0.z; n[3] = n0.w;
       if (cnt > 4) {
-        const float4 n1 = normals4(key, q0 + 1, seg, c2);
+        const float4 n1 = normals4(key, q0 + 1, seg, c2, c3);
         n[4] = n1.x; n[5] = n1.y; n[6] = n1.z; n[7] = n1.w;
       } else {
         n[4] = n[5] = n[6] = n[7] = 0.f;
@@ -265,6 +266,20 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
     }
 
     const uint64_t g = (uint64_t)seg * p.L + e0;
+    if (p.recompute) {
+      // independent benign recompute: the fp16 output, stored as fp32
+      if (cnt == 8 && (g & 7) == 0) {
+        float4 *r4 = reinterpret_cast<float4 *>(refs + g);
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = __half2float(__float2half_rn(h[k]));
+        r4[0] = make_float4(v[0], v[1], v[2], v[3]);
+        r4[1] = make_float4(v[4], v[5], v[6], v[7]);
+      } else {
+        for (int k = 0; k < cnt; ++k) refs[g + k] = __half2float(__float2half_rn(h[k]));
+      }
+      continue;
+    }
     if (cnt == 8 && (g & 7) == 0) {
       float4 *r4 = reinterpret_cast<float4 *>(refs + g);
       r4[0] = make_float4(a[0], a[1], a[2], a[3]);
@@ -286,6 +301,20 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
       }
     }
   }
+}
+
+// ----------------------------------------------------------------- random baseline
+// Sec. 4.5: every score replaced by Uniform(0, 1).  Thread per (config,
+// canary); score s = (x >> 8) 2^-24 with x word s of aux stream
+// (RANDOM, canary) of config id config_id0 + c.
+__global__ void random_scores_kernel(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
+                                     uint32_t S, float *__restrict__ out) {
+  const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= (uint64_t)C * N) return;
+  const uint32_t c = (uint32_t)(t / N), n = (uint32_t)(t % N);
+  AuxWords w = aux_words(seed, kAuxRandom, n, config_id0 + c);
+  float *o = out + t * S;
+  for (uint32_t s = 0; s < S; ++s) o[s] = (float)(aux_next(w) >> 8) * 0x1p-24f;
 }
 
 // ----------------------------------------------------------------- test views
@@ -364,6 +393,15 @@ cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int
   const uint64_t grid = blocks_needed < resident * 4 ? blocks_needed : resident * 4;
   gen_materialise_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, outlier_mask, flip_mask,
                                                                      coef, acts, refs);
+  // (in recompute mode acts is unused and refs receives the recompute)
+  return cudaGetLastError();
+}
+
+cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
+                                 uint32_t S, float *out, cudaStream_t stream) {
+  const uint64_t n = (uint64_t)C * N;
+  random_scores_kernel<<<(unsigned)((n + 127) / 128), 128, 0, stream>>>(seed, config_id0, C, N, S,
+                                                                        out);
   return cudaGetLastError();
 }
 

@@ -91,3 +91,39 @@ def test_control_no_benign_flag(cg):
     cg.cg_make_control_labels(torch.from_numpy(labels).cuda(), seed=1, status=st)
     status, word = cg.cg_read_status(st)
     assert status == 8 and word == cg.DEVFLAG_NO_BENIGN
+
+
+@pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
+    (1, 1, 2, 1, 0, None), (5, 7, 4, 1, 0, None), (3, 64, 16, 1, 0, 3), (4, 9, 32, 3, 2, 5),
+    (2, 256, 16, 1, 0, None), (2, 1000, 16, 2, 1, 7), (324, 64, 16, 1, 0, None), (1, 1, 1000, 10, 3, 6),
+])
+def test_pooled_matches_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
+    import torch
+    scores, labels = SI.score_arrays(C, N, S, seed=C * 7 + N + S, n_malicious=n_mal,
+                                     tie_levels=ties, excluded=excluded)
+    g = cg.cg_auroc_pooled(torch.from_numpy(scores).cuda(), torch.from_numpy(labels).cuda())
+    o = orc.auroc_pooled(scores, labels)
+    for k in ("u2", "n_mal", "n_ben"):
+        assert np.array_equal(g[k].cpu().numpy(), o[k]), k
+    assert np.array_equal(g["auroc"].cpu().numpy().view(np.uint64), o["auroc"].view(np.uint64))
+
+
+def test_pooled_signed_zero_and_inf(cg, orc):
+    import torch
+    scores = np.array([[[0.0, -0.0, np.inf, -np.inf, 1.0, -1.0]]], np.float32)
+    labels = np.array([[[1, 0, 1, 0, 0, 1]]], np.int8)
+    g = cg.cg_auroc_pooled(torch.from_numpy(scores).cuda(), torch.from_numpy(labels).cuda())
+    o = orc.auroc_pooled(scores, labels)
+    assert g["u2"].item() == o["u2"][0]
+    assert g["auroc"].item() == o["auroc"][0]
+
+
+def test_pooled_nan_flag(cg, orc):
+    import torch
+    scores, labels = SI.score_arrays(2, 5, 4, seed=3)
+    scores[1, 2, 1] = np.nan
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = cg.cg_auroc_pooled(torch.from_numpy(scores).cuda(), torch.from_numpy(labels).cuda(), status=st)
+    o = orc.auroc_pooled(scores, labels, allow_nan=True)
+    assert cg.cg_read_status(st)[0] == 4
+    assert np.array_equal(g["u2"].cpu().numpy(), o["u2"])

@@ -1,0 +1,87 @@
+"""GPU parity of the reference conditions (Sec. 4.5) and the noisy-reference
+ablation (Sec. 4.4): random-baseline scores bit-exact, the independent benign
+recompute within 1 fp16 ulp of the oracle's, and the detection outcomes of
+Table 1 (ceiling 1.000, noisy reference 1.000, random baseline near 0.5)."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import seeded_inputs as SI
+from tests._cmp import half_ulp_distance
+
+pytestmark = pytest.mark.gpu
+PAPER = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "paper_values.json")))
+
+
+@pytest.fixture(scope="module")
+def cg():
+    torch = pytest.importorskip("torch")
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_19490_gb300 as m
+    m.build()
+    return m
+
+
+@pytest.mark.parametrize("C,N,S,cid0", [(1, 1, 1, 0), (3, 7, 5, 9), (324, 64, 16, 0), (2, 100, 33, 1000)])
+def test_random_scores_bit_exact(cg, orc, C, N, S, cid0):
+    g = cg.cg_random_scores(123, C, N, S, config_id0=cid0).cpu().numpy()
+    assert np.array_equal(g, orc.random_scores(123, C, N, S, config_id0=cid0))
+
+
+def test_random_baseline_auroc_matches_oracle(cg, orc):
+    import torch
+    C, N, S = 200, 100, 4
+    sc = cg.cg_random_scores(9, C, N, S)
+    labels = np.zeros((C, N, S), np.int8)
+    labels[:, :, 1] = 1
+    g = cg.cg_auroc(sc, torch.from_numpy(labels).cuda())["auroc"].cpu().numpy()
+    o = orc.auroc(orc.random_scores(9, C, N, S), labels)["auroc"]
+    assert np.array_equal(g, o)
+    assert abs(g.mean() - PAPER["random_baseline"]["mean"]) < 0.01
+
+
+RECOMPUTE_CASES = {
+    "tiny": SI.TINY,
+    "paper_shape_small": SI.shrink(SI.PAPER_SHAPE, n_canaries=4, tokens=6),
+    "snr_step": SI.shrink(SI.snr_configs()[3], n_canaries=2, tokens=2, hidden=1024),
+    "ragged": SI.shrink(SI.TINY, hidden=100, tokens=3, n_outlier=3),
+}
+
+
+@pytest.mark.parametrize("name", sorted(RECOMPUTE_CASES))
+@pytest.mark.parametrize("replica", [0, 1, 7])
+def test_recompute_matches_oracle(cg, orc, name, replica):
+    cfg = RECOMPUTE_CASES[name]
+    g = cg.cg_generate_recompute(cg.PipelineDesc.from_config(cfg), replica).cpu().numpy()
+    o = orc.generate_recompute(orc.desc_from_dict(cfg), replica)
+    d = half_ulp_distance(g.astype(np.float16).view(np.uint16), o.astype(np.float16).view(np.uint16))
+    assert np.array_equal(g.astype(np.float16).astype(np.float32), g)   # fp16 values
+    assert d.max() <= 1 and (d > 0).mean() < 1e-2
+
+
+def test_recompute_replica0_equals_live(cg):
+    cfg = SI.shrink(SI.PAPER_SHAPE, n_canaries=4, tokens=6)
+    desc = cg.PipelineDesc.from_config(cfg)
+    acts, _, _ = cg.cg_generate_pipeline(desc)
+    rec = cg.cg_generate_recompute(desc, 0)
+    benign = [s for s in range(cfg["n_shards"]) if s not in cfg["malicious"]]
+    assert np.array_equal(rec.cpu().numpy()[benign], acts.float().cpu().numpy()[benign])
+
+
+@pytest.mark.parametrize("tamper,param", [(SI.TAMPER_ADDITIVE, 0.05), (SI.TAMPER_SIGNFLIP_FULL, 0.0),
+                                          (SI.TAMPER_SCALE, 1.10)])
+def test_ceiling_and_noisy_reference_detect(cg, tamper, param):
+    """Table 1: the recompute ceiling and the noisy-reference ablation both
+    reach A-hat = 1.000 with the relative-L2 mismatch."""
+    cfg = SI.shrink(SI.PAPER_SHAPE, tamper=tamper, tamper_param=param)
+    desc = cg.PipelineDesc.from_config(cfg)
+    acts, refs, labels = cg.cg_generate_pipeline(desc)
+    S, N = cfg["n_shards"], cfg["n_canaries"]
+    for replica in (1, 2):          # noisy reference, recompute ceiling
+        rec = cg.cg_generate_recompute(desc, replica)
+        sc = cg.cg_drift_scores(acts, rec, S, N)
+        A = cg.cg_auroc(sc[0][None].contiguous(), labels[None])["auroc"].item()
+        assert A == PAPER["full_detector_auroc"]["value"]

@@ -167,3 +167,41 @@ def test_control_auroc_near_half(orc):
     lo, hi = PAPER["control_acceptance"]["interval"]
     assert lo <= float(np.mean(vals)) <= hi
     assert orc.auroc(sc[None], labels[None])["auroc"][0] == 1.0
+
+
+# --------------------------------------------------------------------------
+# Pooled Mann-Whitney (all canaries of a configuration in one pool)
+
+def test_pooled_matches_scipy_and_pairs(orc):
+    stats = pytest.importorskip("scipy.stats")
+    for seed, ties, nm, ex in [(1, None, 1, 0), (2, 4, 2, 1), (3, 3, 3, 0)]:
+        scores, labels = SI.score_arrays(3, 11, 7, seed=seed, n_malicious=nm, tie_levels=ties,
+                                         excluded=ex)
+        res = orc.auroc_pooled(scores, labels)
+        for c in range(3):
+            m, l = scores[c].ravel(), labels[c].ravel()
+            U = stats.mannwhitneyu(m[l == 1], m[l == 0], alternative="two-sided").statistic
+            assert res["u2"][c] == round(2 * U)
+            assert res["n_mal"][c] == (l == 1).sum() and res["n_ben"][c] == (l == 0).sum()
+            exact = Fraction(int(res["u2"][c]), 2 * int(res["n_mal"][c]) * int(res["n_ben"][c]))
+            assert res["auroc"][c] == float(exact)
+
+
+def test_pooled_equals_per_canary_when_one_canary(orc):
+    scores, labels = SI.score_arrays(4, 1, 9, seed=8, n_malicious=2, tie_levels=3)
+    assert np.array_equal(orc.auroc_pooled(scores, labels)["u2"],
+                          orc.auroc(scores, labels)["u2"][:, 0])
+
+
+def test_pooled_invariants(orc):
+    scores, labels = SI.score_arrays(3, 5, 6, seed=4, n_malicious=1)
+    base = orc.auroc_pooled(scores, labels)
+    neg = orc.auroc_pooled(-scores, labels)
+    assert np.array_equal(neg["u2"], 2 * base["n_mal"] * base["n_ben"] - base["u2"])
+    assert np.allclose(neg["auroc"], 1.0 - base["auroc"], rtol=0, atol=1e-15)
+    sep = np.where(labels == 1, scores + 2.0, scores).astype(np.float32)
+    assert np.all(orc.auroc_pooled(sep, labels)["auroc"] == 1.0)
+    nan = scores.copy()
+    nan[0, 0, 0] = np.nan
+    with pytest.raises(Exception):
+        orc.auroc_pooled(nan, labels)
