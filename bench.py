@@ -67,6 +67,9 @@ def parse_args(argv=None):
     p.add_argument("--cpu-seconds", type=float, default=10.0,
                    help="target duration of the timed CPU-oracle sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--study", default=None, choices=sorted(SI.STUDIES),
+                   help="run a whole study (generate + score + rank every configuration) and "
+                        "report configurations/s instead of the default step")
     return p.parse_args(argv)
 
 
@@ -530,6 +533,145 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
     return out
 
 
+# ----------------------------------------------------------------------------- studies
+
+STUDY_METRIC = "AUROC configs/sec (whole study: generate, score and rank every configuration)"
+
+
+def study_pass(cg, torch, configs, dev, bufs, res):
+    """Every configuration of a study on the device: generate, drift scores,
+    control labels, per-canary AUROC of rel_l2 / max_abs / cos_dev and of the
+    control, pooled AUROC of rel_l2.  res[c] = those five A-hat values."""
+    for c, cfg in enumerate(configs):
+        S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
+        E = S * N * L
+        desc = cg.PipelineDesc.from_config(cfg)
+        acts = bufs["acts"][:E].view(S, N, L)
+        refs = bufs["refs"][:E].view(S, N, L)
+        labels = bufs["labels"][:N * S].view(1, N, S)
+        ctrl = bufs["ctrl"][:N * S].view(1, N, S)
+        cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"], status=bufs["status"])
+        scores = bufs["scores"][:3 * N * S].view(3, N, S)
+        cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"], status=bufs["status"])
+        cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
+                                  status=bufs["status"])
+        u2 = bufs["u2"][:N].view(1, N)
+        for k in range(3):
+            cg.cg_auroc(scores[k].view(1, N, S), labels, u2=u2, auroc=res[c, k:k + 1],
+                        want_counts=False, status=bufs["status"])
+        cg.cg_auroc(scores[0].view(1, N, S), ctrl, u2=u2, auroc=res[c, 3:4], want_counts=False,
+                    status=bufs["status"])
+        cg.cg_auroc_pooled(scores[0].view(1, N, S), labels, u2=bufs["pu2"], n_mal=bufs["pnm"],
+                           n_ben=bufs["pnb"], auroc=res[c, 4:5], status=bufs["status"])
+
+
+def run_study(args, ranks: Ranks):
+    import torch
+    import paper_2607_19490_gb300 as cg
+
+    torch.cuda.set_device(ranks.local)
+    cg.build()
+    configs = [rank_config(c, ranks.rank) for c in SI.STUDIES[args.study]()]
+    dev = torch.device("cuda", ranks.local)
+    stream = torch.cuda.current_stream()
+    maxE = max(SI.n_elements(c) for c in configs)
+    maxNS = max(c["n_canaries"] * c["n_shards"] for c in configs)
+    maxN = max(c["n_canaries"] for c in configs)
+    gws = max(cg.cg_generate_workspace_size(cg.PipelineDesc.from_config(c)) for c in configs)
+    dws = max(cg.cg_drift_workspace_size(c["n_shards"], c["n_canaries"],
+                                         c["tokens"] * c["hidden"]) for c in configs)
+    bufs = {
+        "acts": torch.empty(maxE, dtype=torch.float16, device=dev),
+        "refs": torch.empty(maxE, dtype=torch.float32, device=dev),
+        "labels": torch.empty(maxNS, dtype=torch.int8, device=dev),
+        "ctrl": torch.empty(maxNS, dtype=torch.int8, device=dev),
+        "scores": torch.empty(3 * maxNS, dtype=torch.float32, device=dev),
+        "u2": torch.empty(maxN, dtype=torch.int64, device=dev),
+        "pu2": torch.empty(1, dtype=torch.int64, device=dev),
+        "pnm": torch.empty(1, dtype=torch.int64, device=dev),
+        "pnb": torch.empty(1, dtype=torch.int64, device=dev),
+        "gws": torch.empty(gws, dtype=torch.uint8, device=dev),
+        "dws": torch.empty(dws, dtype=torch.uint8, device=dev),
+        "status": torch.zeros(1, dtype=torch.int32, device=dev),
+    }
+    res = torch.empty((len(configs), 5), dtype=torch.float64, device=dev)
+    for _ in range(max(1, args.warmup)):
+        study_pass(cg, torch, configs, dev, bufs, res)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(ranks.local)
+    clocks.start()
+    ranks.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(1, args.steps)
+    e0.record(stream)
+    for _ in range(reps):
+        study_pass(cg, torch, configs, dev, bufs, res)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    clk = clocks.stop()
+    ms = ranks.max(e0.elapsed_time(e1)) / reps
+    st, word = cg.cg_read_status(bufs["status"])
+    if st != 0:
+        raise RuntimeError(f"device status {word} during the study")
+    A = res.cpu().numpy()
+    total_cfg = ranks.sum(float(len(configs)))
+    elems = ranks.sum(float(sum(SI.n_elements(c) for c in configs)))
+
+    cpu = None
+    if ranks.rank == 0 and ranks.world == 1 and not args.no_cpu_baseline:
+        cpu = study_oracle_baseline(configs, args.cpu_seconds)
+    if ranks.rank != 0:
+        return
+    names = ["rel_l2", "max_abs", "cos_dev", "control", "pooled_rel_l2"]
+    summary = {n: {"min": float(np.nanmin(A[:, k])), "mean": float(np.nanmean(A[:, k])),
+                   "max": float(np.nanmax(A[:, k])), "n_equal_1": int((A[:, k] == 1.0).sum())}
+               for k, n in enumerate(names)}
+    line = {
+        "metric": STUDY_METRIC, "value": total_cfg / (ms / 1e3), "unit": "configs/s",
+        "n_gpus": ranks.world, "steps": reps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": f"study '{args.study}': {len(configs)} configurations",
+                   "elements_per_pass": elems,
+                   "step": "per configuration: generate (4 kernels), drift (2), control labels, "
+                           "3 + 1 per-canary AUROC, 1 pooled AUROC"},
+        "elements_per_s": elems / (ms / 1e3),
+        "auroc_summary": summary,
+        "per_config_auroc": {n: [round(float(x), 6) for x in A[:, k]] for k, n in enumerate(names)},
+        "cpu_baseline": cpu,
+        "gpu_launches": 12 * len(configs) * reps,
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def study_oracle_baseline(configs, seconds):
+    """The fp64 oracle on a bounded sample of the study: its configurations in
+    order, each with its canaries cut to at most 8, until `seconds` pass."""
+    from oracle import oracle as O
+    O.build()
+    threads = O.max_threads()
+    done, t0 = 0, time.perf_counter()
+    for cfg in configs:
+        sub = SI.shrink(cfg, n_canaries=min(8, cfg["n_canaries"]))
+        D = O.desc_from_dict(sub)
+        acts, refs, labels = O.generate_pipeline(D, n_threads=threads)
+        sc = O.drift_scores(acts, refs, sub["n_shards"], sub["n_canaries"], n_threads=threads)
+        for k in range(3):
+            O.auroc(sc[k].astype(np.float32)[None], labels[None])
+        O.auroc_pooled(sc[0].astype(np.float32)[None], labels[None])
+        done += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    el = time.perf_counter() - t0
+    frac = min(8, configs[0]["n_canaries"]) / configs[0]["n_canaries"]
+    return {"value": done * frac / el, "unit": "configs/s", "cores": threads, "kind": "oracle",
+            "sample": f"first {done} configurations with at most 8 canaries each (generate + "
+                      f"drift + AUROC in fp64), scaled to full canary counts by {frac:.3f}, "
+                      f"{el:.1f} s"}
+
+
 def main(argv=None):
     args = parse_args(argv)
     ranks = Ranks()
@@ -540,6 +682,9 @@ def main(argv=None):
         return 0
     ranks.init("nccl")
     try:
+        if args.study:
+            run_study(args, ranks)
+            return 0
         run_ours(args, ranks)
     finally:
         ranks.close()

@@ -174,3 +174,77 @@ def score_arrays(C, N, S, seed, n_malicious=1, tie_levels=None, excluded=0):
             labels[c, n, perm[:n_malicious]] = 1
             labels[c, n, perm[n_malicious:n_malicious + excluded]] = -1
     return scores, labels
+
+
+# --------------------------------------------------------------------------
+# Substudies around the paper's anchor (Sec. 4.4: Gaussian tamper eps = 0.05,
+# full mechanism, sigma_hw = 0.002, three seeds), at the paper's experiment
+# shape (k = 12, d = 768, n = 100, T = 48).
+
+SUBSTUDY_SEEDS = (5, 6, 7)
+
+
+def anchor(**over):
+    return shrink(PAPER_SHAPE, **over)
+
+
+def collusion_positions(k, c):
+    """c colluders spaced uniformly over k stages: 1-based floor(j k / (c+1)),
+    j = 1..c, as 0-based ids (c = 1 gives floor(k/2), the main experiment's i*)."""
+    return tuple((j * k) // (c + 1) - 1 for j in range(1, c + 1))
+
+
+def collusion_configs(seeds=SUBSTUDY_SEEDS):
+    return [anchor(malicious=collusion_positions(12, c), seed=sd, config_id=100 + 10 * c + i)
+            for c in (1, 2, 3, 4) for i, sd in enumerate(seeds)]
+
+
+POSITION_FRACTIONS = (0.0, 0.25, 0.5, 0.75, 1.0)
+
+
+def position_configs(seeds=SUBSTUDY_SEEDS):
+    """i* at five fractions f of the pipeline: 0-based floor(f (k-1) + 1/2)."""
+    out = []
+    for j, f in enumerate(POSITION_FRACTIONS):
+        pos = int(f * 11 + 0.5)
+        out += [anchor(malicious=(pos,), seed=sd, config_id=200 + 10 * j + i)
+                for i, sd in enumerate(seeds)]
+    return out
+
+
+FRONTIER_EPS = (0.10, 0.05, 0.02, 0.01, 0.005, 0.002, 0.001)
+
+
+def frontier_configs(seeds=SUBSTUDY_SEEDS):
+    """eps from 0.10 down to 0.001 on a 1-2-5 grid at the fixed floor sigma_hw = 0.002."""
+    return [anchor(tamper_param=e, seed=sd, config_id=300 + 10 * j + i)
+            for j, e in enumerate(FRONTIER_EPS) for i, sd in enumerate(seeds)]
+
+
+DEPTHS = (2, 4, 6, 8, 10, 12)
+
+
+def depth_configs(seeds=SUBSTUDY_SEEDS):
+    """k in {2, ..., 12} stages with i* = floor(k/2) (1-based)."""
+    return [anchor(n_shards=k, malicious=(k // 2 - 1,), seed=sd, config_id=400 + 10 * j + i)
+            for j, k in enumerate(DEPTHS) for i, sd in enumerate(seeds)]
+
+
+PAPER_SNR_SIGMAS = (0.002, 0.005, 0.01, 0.02, 0.05, 0.1, 0.2)
+
+
+def paper_snr_configs(seeds=SUBSTUDY_SEEDS):
+    """The paper's own noise-floor substudy: sigma_hw from 0.002 to 0.2 against eps = 0.05."""
+    return [anchor(benign_sigma=sg, seed=sd, config_id=500 + 10 * j + i)
+            for j, sg in enumerate(PAPER_SNR_SIGMAS) for i, sd in enumerate(seeds)]
+
+
+STUDIES = {
+    "factorial": factorial_configs,
+    "snr": snr_configs,
+    "collusion": collusion_configs,
+    "position": position_configs,
+    "frontier": frontier_configs,
+    "depth": depth_configs,
+    "paper_snr": paper_snr_configs,
+}
