@@ -67,6 +67,8 @@ def parse_args(argv=None):
     p.add_argument("--cpu-seconds", type=float, default=10.0,
                    help="target duration of the timed CPU-oracle sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--drift-algo", default="auto", choices=["auto", "stream", "bulk", "bulk2"],
+                   help="drift kernel (cg_drift_scores_ex); auto = cg_drift_scores")
     p.add_argument("--study", default=None, choices=sorted(SI.STUDIES),
                    help="run a whole study (generate + score + rank every configuration) and "
                         "report configurations/s instead of the default step")
@@ -334,11 +336,14 @@ def run_ours(args, ranks: Ranks):
     auroc = torch.empty((2,), dtype=torch.float64, device=dev)
     launches_per_step = 5          # drift partial + finalize, control labels, 2 x AUROC
 
+    algo = {"auto": None, "stream": cg.DRIFT_STREAM, "bulk": cg.DRIFT_BULK,
+            "bulk2": cg.DRIFT_BULK_2CTA}[args.drift_algo]
+
     def step(i, ev=None):
         if ev is not None:
             ev[0].record(stream)
         cg.cg_drift_scores(acts, refs, S, N, scores=scores, stat_stride=N * S, ws=dws,
-                           status=status)
+                           status=status, algo=algo)
         if ev is not None:
             ev[1].record(stream)
         cg.cg_make_control_labels(labels, seed=1000 + i, ctrl=ctrl, status=status)
@@ -378,7 +383,12 @@ def run_ours(args, ranks: Ranks):
     peak, peak_kind = measured_peaks()
     drift_avg_ms = statistics.mean(drift_ms)
     achieved = E * BYTES_PER_ELEMENT / (drift_avg_ms / 1e3) / 1e9
-    traffic = recorded_traffic("drift.cu", f"drift_partial_kernel_{args.workload}.txt")
+    # cg_drift_scores picks the TMA bulk pipeline for device-resident inputs
+    # whose segments are a multiple of 8 elements
+    drift_kernel = ("drift_partial_kernel" if args.drift_algo == "stream" or L % 8
+                    else "drift_bulk_kernel")
+    traffic = (recorded_traffic("drift.cu", f"{drift_kernel}_{args.workload}.txt")
+               if args.drift_algo in ("auto", "stream", "bulk") else None)
 
     # ---- AUROC batches (configs/s): the factorial batch and a stress batch
     auroc_rates = auroc_batches(cg, torch, dev, stream)
@@ -420,7 +430,7 @@ def run_ours(args, ranks: Ranks):
             "step": "drift scores (2 kernels) + control labels + AUROC true and control",
         },
         "roofline": {
-            "kernel": "drift_partial_kernel (+ drift_finalize_kernel inside the same events)",
+            "kernel": drift_kernel + " (+ drift_finalize_kernel inside the same events)",
             "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
             "traffic": traffic,

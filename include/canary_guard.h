@@ -196,6 +196,28 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
                           uint64_t stat_stride, void *d_ws, size_t ws_bytes,
                           int32_t *d_status, cg_stream_t stream);
 
+/* Kernel choice for cg_drift_scores_ex. */
+typedef enum {
+  CG_DRIFT_AUTO = 0,       /* CG_DRIFT_BULK when both inputs are device memory and
+                              seg_len % 8 == 0, else CG_DRIFT_STREAM (cg_drift_scores) */
+  CG_DRIFT_STREAM = 1,     /* register-streaming kernel, any seg_len */
+  CG_DRIFT_BULK = 2,       /* TMA bulk-copy pipeline, 8 shared-memory stages, 1 block per SM;
+                              needs device memory and seg_len % 8 == 0
+                              (else CG_ERR_UNSUPPORTED) */
+  CG_DRIFT_BULK_2CTA = 3   /* TMA bulk-copy pipeline, 4 stages, 2 blocks per SM; same need */
+} cg_drift_algo;
+
+/*
+ * cg_drift_scores with an explicit kernel choice (same results up to the
+ * order of fp32 additions).  The bulk-copy kernels report a wait that gave
+ * up as CG_DEVFLAG_TIMEOUT in d_status.
+ */
+cg_status cg_drift_scores_ex(const uint16_t *d_acts, const float *d_refs,
+                             uint32_t n_shards, uint32_t n_canaries,
+                             uint64_t seg_len, float *d_scores,
+                             uint64_t stat_stride, void *d_ws, size_t ws_bytes,
+                             int32_t *d_status, int32_t algo, cg_stream_t stream);
+
 /*
  * cg_drift_scores with the live activations in pinned host memory: the
  * drift kernel reads h_acts directly over the host-GPU link (one pass, no

@@ -20,7 +20,7 @@ __all__ = [
     "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
     "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
-    "cg_drift_scores_host", "cg_drift_scores_noalloc",
+    "cg_drift_scores_ex", "cg_drift_scores_host", "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
     "cg_random_scores", "cg_auroc_pooled",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
@@ -34,6 +34,7 @@ STATUS_NAMES = {0: "CG_OK", 1: "CG_ERR_INVALID_ARG", 2: "CG_ERR_ALIGNMENT", 3: "
 NOISE_MULT, NOISE_PAPER = 0, 1
 TAMPER_ADDITIVE, TAMPER_SIGNFLIP_CHANNELS, TAMPER_SIGNFLIP_FULL, TAMPER_SCALE = 0, 1, 2, 3
 DEVFLAG_NAN_SCORE, DEVFLAG_TIMEOUT, DEVFLAG_NO_BENIGN = 1, 2, 4
+DRIFT_AUTO, DRIFT_STREAM, DRIFT_BULK, DRIFT_BULK_2CTA = 0, 1, 2, 3
 
 
 class CgError(RuntimeError):
@@ -98,6 +99,7 @@ def load() -> ctypes.CDLL:
             "cg_generate_recompute": ([ctypes.POINTER(PipelineDesc), u32, P, P, sz, P, P], ctypes.c_int),
             "cg_random_scores": ([u64, u32, u32, u32, u32, P, P], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
+            "cg_drift_scores_ex": ([P, P, u32, u32, u64, P, u64, P, sz, P, ctypes.c_int32, P], ctypes.c_int),
             "cg_drift_scores_host": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_noalloc": ([P, P, u32, u32, u64, P, u64, P, P], ctypes.c_int),
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
@@ -260,8 +262,9 @@ def cg_drift_workspace_size(n_shards, n_canaries, seg_len) -> int:
 
 
 def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=None, ws=None,
-                    status=None, stream=None):
-    """Drift scores [3][N][S] (rel_l2, max_abs, cos_dev) of acts fp16 / refs fp32 [S][N][L]."""
+                    status=None, stream=None, algo=None):
+    """Drift scores [3][N][S] (rel_l2, max_abs, cos_dev) of acts fp16 / refs fp32 [S][N][L].
+    `algo` (DRIFT_*) selects the kernel through cg_drift_scores_ex; None calls cg_drift_scores."""
     torch = _torch()
     _cuda(acts, "acts", (torch.float16,))
     _cuda(refs, "refs", (torch.float32,))
@@ -284,9 +287,15 @@ def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=N
         raise ValueError("scores must hold 2 * stat_stride + N * S floats")
     if ws.numel() < cg_drift_workspace_size(n_shards, n_canaries, seg_len):
         raise ValueError("workspace smaller than cg_drift_workspace_size")
-    _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
-                                  _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
-                                  _stream(stream)), "cg_drift_scores")
+    if algo is None:
+        _check(load().cg_drift_scores(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
+                                      _ptr(scores), stat_stride, _ptr(ws), ws.numel(), _ptr(status),
+                                      _stream(stream)), "cg_drift_scores")
+    else:
+        _check(load().cg_drift_scores_ex(_ptr(acts), _ptr(refs), n_shards, n_canaries, seg_len,
+                                         _ptr(scores), stat_stride, _ptr(ws), ws.numel(),
+                                         _ptr(status), int(algo), _stream(stream)),
+               "cg_drift_scores_ex")
     return scores
 
 

@@ -46,6 +46,16 @@ inline bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
 
 inline cg_status from_cuda(cudaError_t e) { return e == cudaSuccess ? CG_OK : CG_ERR_CUDA; }
 
+// true for memory allocated on a device (cudaMalloc and friends)
+bool is_device_memory(const void *p) {
+  cudaPointerAttributes attr;
+  if (cudaPointerGetAttributes(&attr, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return attr.type == cudaMemoryTypeDevice;
+}
+
 cg_status check_desc(const cg_pipeline_desc *d) {
   if (!d) return CG_ERR_INVALID_ARG;
   if (d->n_shards < 1 || d->hidden < 1 || d->n_canaries < 1 || d->tokens < 1)
@@ -212,8 +222,17 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs, uint32_t 
                           uint32_t n_canaries, uint64_t seg_len, float *d_scores,
                           uint64_t stat_stride, void *d_ws, size_t ws_bytes, int32_t *d_status,
                           cg_stream_t stream) {
+  return cg_drift_scores_ex(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores, stat_stride,
+                            d_ws, ws_bytes, d_status, CG_DRIFT_AUTO, stream);
+}
+
+cg_status cg_drift_scores_ex(const uint16_t *d_acts, const float *d_refs, uint32_t n_shards,
+                             uint32_t n_canaries, uint64_t seg_len, float *d_scores,
+                             uint64_t stat_stride, void *d_ws, size_t ws_bytes, int32_t *d_status,
+                             int32_t algo, cg_stream_t stream) {
   if (!d_acts || !d_refs || !d_scores || n_shards == 0 || n_canaries == 0 || seg_len == 0)
     return CG_ERR_INVALID_ARG;
+  if (algo < CG_DRIFT_AUTO || algo > CG_DRIFT_BULK_2CTA) return CG_ERR_INVALID_ARG;
   const uint64_t n_seg = (uint64_t)n_shards * n_canaries;
   if (stat_stride < n_seg) return CG_ERR_INVALID_ARG;
   if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
@@ -222,9 +241,16 @@ cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs, uint32_t 
     return CG_ERR_ALIGNMENT;
   if (!d_ws || ws_bytes < cg::drift_ws_bytes(n_seg, seg_len)) return CG_ERR_WORKSPACE;
   if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
-  (void)d_status;   // the streaming path has no device-side failure mode
-  return from_cuda(cg::launch_drift(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores,
-                                    stat_stride, d_ws, (cudaStream_t)stream));
+  // The bulk-copy pipelines take device memory only (8-element aligned
+  // segments); anything else streams through registers.
+  const bool bulk_ok = cg::drift_bulk_eligible(d_acts, d_refs, seg_len) &&
+                       is_device_memory(d_acts) && is_device_memory(d_refs);
+  if ((algo == CG_DRIFT_BULK || algo == CG_DRIFT_BULK_2CTA) && !bulk_ok)
+    return CG_ERR_UNSUPPORTED;
+  if (algo == CG_DRIFT_AUTO) algo = bulk_ok ? CG_DRIFT_BULK : CG_DRIFT_STREAM;
+  return from_cuda(cg::launch_drift_algo(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores,
+                                         stat_stride, d_ws, d_status, algo,
+                                         (cudaStream_t)stream));
 }
 
 cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs, uint32_t n_shards,
@@ -241,9 +267,9 @@ cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs, uint
     return CG_ERR_INVALID_ARG;
   }
   if (attr.type != cudaMemoryTypeHost || attr.devicePointer == nullptr) return CG_ERR_INVALID_ARG;
-  return cg_drift_scores(static_cast<const uint16_t *>(attr.devicePointer), d_refs, n_shards,
-                         n_canaries, seg_len, d_scores, stat_stride, d_ws, ws_bytes, d_status,
-                         stream);
+  return cg_drift_scores_ex(static_cast<const uint16_t *>(attr.devicePointer), d_refs, n_shards,
+                            n_canaries, seg_len, d_scores, stat_stride, d_ws, ws_bytes, d_status,
+                            CG_DRIFT_STREAM, stream);
 }
 
 cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,

@@ -39,6 +39,11 @@ cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, ui
                          uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
                          cudaStream_t stream);
 
+bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len);
+cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                              uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
+                              int32_t *status, int algo, cudaStream_t stream);
+
 // Work-item capacity of the fixed scratch array used by cg_drift_scores_noalloc.
 constexpr uint64_t kNoallocDriftItems = 262144;
 cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,

@@ -197,7 +197,285 @@ __global__ void drift_finalize_kernel(const float4 *__restrict__ partials, uint6
   scores[2 * stat_stride + o] = (float)cosd;
 }
 
+// ----------------------------------------------------------------- TMA bulk pipeline
+// drift_bulk_kernel: the same work items and per-item float4 partials as
+// drift_partial_kernel, but the bytes are staged through shared memory by
+// the Tensor Memory Accelerator's 1-D bulk copies:
+//   warp 0, lane 0   producer: for every stage (<= kBulkStageElems elements
+//                    of one item) waits for its ring slot to be released,
+//                    arms the slot's `full` mbarrier with the byte count and
+//                    issues two cp.async.bulk copies (fp16 live, fp32 ref).
+//   warps 1..8       consumers: wait on `full`, read the slot (8-byte fp16
+//                    and 16-byte fp32 loads, bank-conflict free), accumulate,
+//                    release the slot on `empty` (one arrival per warp).
+// At the end of an item each consumer warp parks its sums in a
+// double-buffered shared slot and arrives on `red_full`; consumer warp 0
+// waits, adds the eight warps in order and writes the item's partial, then
+// arrives on `red_empty` for that buffer.  Every wait is an mbarrier
+// try_wait loop that gives up after kBulkWaitNs of global-timer time and
+// raises CG_DEVFLAG_TIMEOUT; there is no CTA-wide barrier after the roles
+// split, so an abandoned wait cannot deadlock the block, and the producer
+// waits (bounded) for its copies still in flight before it returns.
+// Requires seg_len % 8 == 0 and 16-byte aligned bases (every copy then
+// starts on a 16-byte boundary and moves a multiple of 16 bytes).
+constexpr int kBulkStageElems = 4096;
+constexpr int kBulkConsumerWarps = 8;
+constexpr int kBulkThreads = 32 * (1 + kBulkConsumerWarps);
+constexpr unsigned long long kBulkWaitNs = 1000000000ull;   // 1 s
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  unsigned long long state;
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
+               : "=l"(state)
+               : "r"(bar), "r"(bytes)
+               : "memory");
+  (void)state;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  unsigned long long state;
+  asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];" : "=l"(state) : "r"(bar) : "memory");
+  (void)state;
+}
+
+// true once the phase with the given parity has completed; false after
+// kBulkWaitNs without completion
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  const unsigned long long t0 = global_ns();
+  for (uint32_t it = 0;; ++it) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    if (done) return true;
+    if ((it & 63u) == 63u && global_ns() - t0 > kBulkWaitNs) return false;
+  }
+}
+
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
+                                         uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+      ::"r"(dst), "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
+}
+
+template <int NS>
+struct BulkSmem {
+  float refs[NS][kBulkStageElems];
+  uint16_t acts[NS][kBulkStageElems];
+  unsigned long long full[NS];
+  unsigned long long empty[NS];
+  unsigned long long red_full[2];
+  unsigned long long red_empty[2];
+  float4 slot[2][kBulkConsumerWarps];
+};
+
+template <int NS>
+__global__ void __launch_bounds__(kBulkThreads)
+drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ refs, uint64_t L,
+                  uint64_t chunks_per_seg, uint64_t n_items, float4 *__restrict__ partials,
+                  int32_t *status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  BulkSmem<NS> &sm = *reinterpret_cast<BulkSmem<NS> *>(smem_raw);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) {
+    for (int i = 0; i < NS; ++i) {
+      mbar_init((uint32_t)__cvta_generic_to_shared(&sm.full[i]), 1);
+      mbar_init((uint32_t)__cvta_generic_to_shared(&sm.empty[i]), kBulkConsumerWarps);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init((uint32_t)__cvta_generic_to_shared(&sm.red_full[b]), kBulkConsumerWarps);
+      mbar_init((uint32_t)__cvta_generic_to_shared(&sm.red_empty[b]), 1);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();   // the only CTA-wide barrier: before the roles split
+
+  if (warp == 0) {
+    // ------------------------------------------------------------- producer
+    if (lane != 0) return;
+    uint32_t stage = 0;
+    bool ok = true;
+    for (uint64_t item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
+      const uint64_t seg = item / chunks_per_seg;
+      const uint64_t ch = item - seg * chunks_per_seg;
+      const uint64_t g0 = seg * L + ch * kDriftChunk;
+      const uint64_t len = min((uint64_t)kDriftChunk, L - ch * kDriftChunk);
+      for (uint64_t off = 0; off < len; off += kBulkStageElems, ++stage) {
+        const uint32_t n = (uint32_t)min((uint64_t)kBulkStageElems, len - off);
+        const int slot = (int)(stage % NS);
+        const uint32_t round = stage / NS;
+        if (round > 0 &&
+            !mbar_wait((uint32_t)__cvta_generic_to_shared(&sm.empty[slot]), (round - 1) & 1u)) {
+          ok = false;
+          break;
+        }
+        const uint32_t fb = (uint32_t)__cvta_generic_to_shared(&sm.full[slot]);
+        mbar_arrive_expect_tx(fb, n * 6u);
+        bulk_g2s((uint32_t)__cvta_generic_to_shared(&sm.acts[slot][0]), acts + g0 + off, n * 2u, fb);
+        bulk_g2s((uint32_t)__cvta_generic_to_shared(&sm.refs[slot][0]), refs + g0 + off, n * 4u, fb);
+      }
+    }
+    if (!ok && status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
+    // before returning, wait (bounded) for the copies still in flight: the
+    // last min(stage, NS) stages issued
+    const uint32_t last = stage;
+    for (uint32_t st = (last > (uint32_t)NS ? last - NS : 0); st < last; ++st) {
+      const int slot = (int)(st % NS);
+      if (!mbar_wait((uint32_t)__cvta_generic_to_shared(&sm.full[slot]), (st / NS) & 1u)) {
+        if (status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
+        break;
+      }
+    }
+    return;
+  }
+
+  // --------------------------------------------------------------- consumers
+  const int cw = warp - 1;                 // consumer warp 0..7
+  const int ct = tid - 32;                 // consumer thread 0..255
+  uint32_t stage = 0, local_item = 0;
+  for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x, ++local_item) {
+    const uint64_t ch = item % chunks_per_seg;
+    const uint64_t len = min((uint64_t)kDriftChunk, L - ch * kDriftChunk);
+    Acc s = {0.f, 0.f, 0.f, 0.f};
+    for (uint64_t off = 0; off < len; off += kBulkStageElems, ++stage) {
+      const uint32_t n = (uint32_t)min((uint64_t)kBulkStageElems, len - off);
+      const int slot = (int)(stage % NS);
+      // every lane waits; the warp leaves together if any lane gave up
+      const bool got = mbar_wait((uint32_t)__cvta_generic_to_shared(&sm.full[slot]),
+                                 (stage / NS) & 1u);
+      if (!__all_sync(0xFFFFFFFFu, got)) {
+        if (lane == 0 && status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
+        return;
+      }
+      const uint2 *a4 = reinterpret_cast<const uint2 *>(&sm.acts[slot][0]);
+      const float4 *r4 = reinterpret_cast<const float4 *>(&sm.refs[slot][0]);
+      for (uint32_t i = ct; i < n / 4; i += 32 * kBulkConsumerWarps) {
+        const uint2 hv = a4[i];
+        const float4 r = r4[i];
+        Acc t = {0.f, 0.f, 0.f, s.m};
+        const float2 h01 = half2_bits_to_float2(hv.x);
+        const float2 h23 = half2_bits_to_float2(hv.y);
+        acc_one(h01.x, r.x, t);
+        acc_one(h01.y, r.y, t);
+        acc_one(h23.x, r.z, t);
+        acc_one(h23.y, r.w, t);
+        s.d += t.d;
+        s.e += t.e;
+        s.a += t.a;
+        s.m = t.m;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive((uint32_t)__cvta_generic_to_shared(&sm.empty[slot]));
+    }
+    // item reduction: warp tree, then warp slots summed in order by consumer warp 0
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      s.d += __shfl_down_sync(0xFFFFFFFFu, s.d, off);
+      s.e += __shfl_down_sync(0xFFFFFFFFu, s.e, off);
+      s.a += __shfl_down_sync(0xFFFFFFFFu, s.a, off);
+      s.m = fmaxf(s.m, __shfl_down_sync(0xFFFFFFFFu, s.m, off));
+    }
+    const int b = (int)(local_item & 1u);
+    const uint32_t use = local_item >> 1;          // how often buffer b was used before
+    if (lane == 0) {
+      if (use > 0 &&
+          !mbar_wait((uint32_t)__cvta_generic_to_shared(&sm.red_empty[b]), (use - 1) & 1u)) {
+        if (status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
+      }
+      sm.slot[b][cw] = make_float4(s.d, s.e, s.a, s.m);
+      mbar_arrive((uint32_t)__cvta_generic_to_shared(&sm.red_full[b]));
+      if (cw == 0) {
+        if (mbar_wait((uint32_t)__cvta_generic_to_shared(&sm.red_full[b]), use & 1u)) {
+          float4 t = sm.slot[b][0];
+          for (int w = 1; w < kBulkConsumerWarps; ++w) {
+            const float4 v = sm.slot[b][w];
+            t.x += v.x;
+            t.y += v.y;
+            t.z += v.z;
+            t.w = fmaxf(t.w, v.w);
+          }
+          partials[item] = t;
+        } else if (status) {
+          atomicOr(status, CG_DEVFLAG_TIMEOUT);
+        }
+        mbar_arrive((uint32_t)__cvta_generic_to_shared(&sm.red_empty[b]));
+      }
+    }
+    __syncwarp();
+  }
+}
+
 }  // namespace
+
+template <int NS>
+static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t seg_len,
+                               uint64_t cps, uint64_t n_items, float4 *partials, int32_t *status,
+                               int sm_count, cudaStream_t stream) {
+  const size_t smem = sizeof(BulkSmem<NS>);
+  cudaError_t err = cudaFuncSetAttribute(drift_bulk_kernel<NS>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  int per_sm = 0;
+  err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, drift_bulk_kernel<NS>, kBulkThreads,
+                                                      smem);
+  if (err != cudaSuccess) return err;
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  uint64_t grid = (uint64_t)sm_count * (uint64_t)per_sm;
+  if (grid > n_items) grid = n_items;
+  drift_bulk_kernel<NS><<<(unsigned)grid, kBulkThreads, smem, stream>>>(acts, refs, seg_len, cps,
+                                                                        n_items, partials, status);
+  return cudaGetLastError();
+}
+
+bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len) {
+  return (seg_len % 8) == 0 && ((uintptr_t)acts % 16) == 0 && ((uintptr_t)refs % 16) == 0;
+}
+
+cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
+                              uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
+                              int32_t *status, int algo, cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  const uint64_t n_seg = (uint64_t)S * N;
+  const uint64_t cps = drift_chunks_per_seg(seg_len);
+  const uint64_t n_items = n_seg * cps;
+  float4 *partials = reinterpret_cast<float4 *>(static_cast<char *>(ws) + kDriftHeader);
+  cudaError_t err;
+  if (algo == CG_DRIFT_BULK) {
+    err = launch_bulk<8>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
+  } else if (algo == CG_DRIFT_BULK_2CTA) {
+    err = launch_bulk<4>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
+  } else {
+    uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
+    if (grid > n_items) grid = n_items;
+    if (grid < 1) grid = 1;
+    drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
+                                                                       n_items, partials);
+    err = cudaGetLastError();
+  }
+  if (err != cudaSuccess) return err;
+  const unsigned fin_threads = 128;
+  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
+  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
+                                                                          scores, stat_stride);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
                          uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,

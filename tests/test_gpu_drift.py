@@ -149,3 +149,43 @@ def test_drift_host_rejects_pageable(cg):
     st = L.cg_drift_scores_host(ctypes.cast(buf, ctypes.c_void_p), fake, 2, 2, 16, fake, 4, fake,
                                 1 << 20, None, None)
     assert st == 1
+
+
+@pytest.mark.parametrize("algo", [1, 2, 3])
+@pytest.mark.parametrize("S,N,L", [(2, 3, 8), (4, 4, 104), (2, 2, 16384), (3, 5, 40000),
+                                   (1, 2, 65536 + 8), (5, 7, 4096), (4, 16, 8192), (2, 3, 4096 * 3 + 8)])
+def test_drift_kernels_match_oracle(cg, orc, algo, S, N, L):
+    """The register-streaming kernel and both TMA bulk-copy pipelines against
+    the oracle; the bulk pipelines' bounded waits never give up."""
+    import torch
+    acts, refs = SI.drift_arrays(S, N, L, seed=S * 31 + N * 7 + L + algo)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = run(cg, acts, refs, S, N, algo=algo, status=st).cpu().numpy()
+    assert cg.cg_read_status(st) == (0, 0)
+    assert_scores_close(g, orc.drift_scores(acts, refs, S, N), what=f"algo {algo}")
+
+
+def test_drift_bulk_rejects_ragged(cg):
+    import torch
+    acts, refs = SI.drift_arrays(2, 2, 12, seed=1)
+    with pytest.raises(cg.CgError) as e:
+        run(cg, acts, refs, 2, 2, algo=cg.DRIFT_BULK)
+    assert e.value.status == 7
+
+
+@pytest.mark.parametrize("algo", [2, 3])
+def test_drift_bulk_full_size_matches_stream(cg, algo):
+    """70B-like workload: the bulk pipelines agree with the streaming kernel."""
+    import torch
+    from tests._cmp import REL_L2_RTOL
+    cfg = SI.SEVENTY_B
+    S, N = cfg["n_shards"], cfg["n_canaries"]
+    acts, refs, _ = cg.cg_generate_pipeline(cg.PipelineDesc.from_config(cfg))
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    a = cg.cg_drift_scores(acts, refs, S, N, algo=1).cpu().numpy()
+    b = cg.cg_drift_scores(acts, refs, S, N, algo=algo, status=st).cpu().numpy()
+    assert cg.cg_read_status(st) == (0, 0)
+    assert np.all(np.abs(a[0] - b[0]) <= 2 * REL_L2_RTOL * np.abs(a[0]))
+    assert np.array_equal(a[1], b[1])
+    del acts, refs
+    torch.cuda.empty_cache()
