@@ -9,6 +9,8 @@
 // Counts are integers (exact in any order); the configuration's A-hat is
 // one fp64 division of exact integers when every canary has the same pair
 // count, else the per-canary ratios added in canary order by one thread.
+#include <climits>
+
 #include "cg_internal.h"
 #include "cg_rng.cuh"
 
@@ -144,6 +146,155 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
           acc = __dadd_rn(acc, __ddiv_rn((double)u2_out[(uint64_t)c * N + n], (double)(2 * nm * nb)));
         }
         A = __ddiv_rn(acc, (double)valid);
+      }
+      auroc[c] = A;
+    }
+    __syncthreads();
+  }
+}
+
+// Small batches (few configurations): the same per-canary counts with one
+// warp per (configuration, canary) across the whole grid, then one block
+// per configuration combines them.  Integer sums make both paths give the
+// same bits.
+__device__ __forceinline__ void canary_counts(const float *m_all, const int8_t *l_all, uint32_t S,
+                                              int lane, long long &g, long long &e, int &nm,
+                                              int &nb, bool &saw_nan) {
+  g = 0;
+  e = 0;
+  if (S <= 32) {
+    const bool in = (uint32_t)lane < S;
+    const float m = in ? m_all[lane] : 0.f;
+    const int l = in ? (int)l_all[lane] : -1;
+    if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
+    int lg = 0, le = 0;
+    for (uint32_t k = 0; k < S; ++k) {
+      const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
+      const int lk = __shfl_sync(0xFFFFFFFFu, l, k);
+      if (l == 1 && lk == 0) {
+        lg += (m > mk);
+        le += (m == mk);
+      }
+    }
+    nm = __popc(__ballot_sync(0xFFFFFFFFu, l == 1));
+    nb = __popc(__ballot_sync(0xFFFFFFFFu, l == 0));
+    g = lg;
+    e = le;
+  } else {
+    int lm = 0, lb = 0;
+    for (uint32_t i = lane; i < S; i += 32) {
+      const float m = m_all[i];
+      const int l = (int)l_all[i];
+      if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
+      lm += (l == 1);
+      lb += (l == 0);
+      if (l != 1) continue;
+      for (uint32_t j = 0; j < S; ++j) {
+        if (l_all[j] != 0) continue;
+        const float mj = m_all[j];
+        g += (m > mj);
+        e += (m == mj);
+      }
+    }
+    nm = lm;
+    nb = lb;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      nm += __shfl_xor_sync(0xFFFFFFFFu, nm, off);
+      nb += __shfl_xor_sync(0xFFFFFFFFu, nb, off);
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    g += __shfl_xor_sync(0xFFFFFFFFu, g, off);
+    e += __shfl_xor_sync(0xFFFFFFFFu, e, off);
+  }
+}
+
+__global__ void __launch_bounds__(kRankThreads)
+auroc_canary_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                    uint64_t n_canaries_total, uint32_t S, int64_t *__restrict__ u2_out,
+                    int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out, int32_t *status) {
+  const int lane = threadIdx.x & 31;
+  const uint64_t warps = (uint64_t)gridDim.x * kRankWarps;
+  bool saw_nan = false;
+  for (uint64_t o = (uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5); o < n_canaries_total;
+       o += warps) {
+    long long g, e;
+    int nm, nb;
+    canary_counts(scores + o * S, labels + o * S, S, lane, g, e, nm, nb, saw_nan);
+    if (lane == 0) {
+      u2_out[o] = 2 * g + e;
+      if (gt_out) gt_out[o] = g;
+      if (eq_out) eq_out[o] = e;
+    }
+  }
+  if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
+    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+}
+
+__global__ void __launch_bounds__(kRankThreads)
+auroc_config_kernel(const int8_t *__restrict__ labels, uint32_t C, uint32_t N, uint32_t S,
+                    const int64_t *__restrict__ u2, double *__restrict__ auroc) {
+  __shared__ long long red[kRankWarps][4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
+    long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
+    for (uint32_t n = tid; n < N; n += kRankThreads) {
+      const int8_t *l = labels + ((uint64_t)c * N + n) * S;
+      long long nm = 0, nb = 0;
+      for (uint32_t s = 0; s < S; ++s) {
+        nm += (l[s] == 1);
+        nb += (l[s] == 0);
+      }
+      const long long pairs = nm * nb;
+      if (pairs > 0) {
+        total += u2[(uint64_t)c * N + n];
+        valid += 1;
+        pmin = min(pmin, pairs);
+        pmax = max(pmax, pairs);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      total += __shfl_down_sync(0xFFFFFFFFu, total, off);
+      valid += __shfl_down_sync(0xFFFFFFFFu, valid, off);
+      pmin = min(pmin, __shfl_down_sync(0xFFFFFFFFu, pmin, off));
+      pmax = max(pmax, __shfl_down_sync(0xFFFFFFFFu, pmax, off));
+    }
+    if (lane == 0) {
+      red[warp][0] = total;
+      red[warp][1] = valid;
+      red[warp][2] = pmin;
+      red[warp][3] = pmax;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < kRankWarps; ++w) {
+        red[0][0] += red[w][0];
+        red[0][1] += red[w][1];
+        red[0][2] = min(red[0][2], red[w][2]);
+        red[0][3] = max(red[0][3], red[w][3]);
+      }
+      const long long T = red[0][0], V = red[0][1];
+      double A;
+      if (V == 0) {
+        A = NAN;
+      } else if (red[0][2] == red[0][3]) {
+        A = __ddiv_rn((double)T, (double)(2 * red[0][2] * V));
+      } else {
+        double acc = 0.0;
+        for (uint32_t n = 0; n < N; ++n) {
+          const int8_t *l = labels + ((uint64_t)c * N + n) * S;
+          long long nm = 0, nb = 0;
+          for (uint32_t s = 0; s < S; ++s) {
+            nm += (l[s] == 1);
+            nb += (l[s] == 0);
+          }
+          if (nm * nb == 0) continue;
+          acc = __dadd_rn(acc, __ddiv_rn((double)u2[(uint64_t)c * N + n], (double)(2 * nm * nb)));
+        }
+        A = __ddiv_rn(acc, (double)V);
       }
       auroc[c] = A;
     }
@@ -333,10 +484,24 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
                          int32_t *status, cudaStream_t stream) {
   DeviceInfo info;
   if (!device_info(&info)) return cudaGetLastError();
-  uint64_t grid = (uint64_t)info.sm_count * 8;
-  if (grid > C) grid = C;
-  auroc_kernel<<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, u2, gt, eq,
-                                                            auroc, status);
+  if ((uint64_t)C >= 2ull * (uint64_t)info.sm_count) {
+    // many configurations: one block each, canaries and combine fused
+    uint64_t grid = (uint64_t)info.sm_count * 8;
+    if (grid > C) grid = C;
+    auroc_kernel<<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, u2, gt, eq,
+                                                              auroc, status);
+    return cudaGetLastError();
+  }
+  // few configurations: spread the canaries over the GPU, then combine
+  const uint64_t total = (uint64_t)C * N;
+  uint64_t blocks = (total + kRankWarps - 1) / kRankWarps;
+  const uint64_t cap = (uint64_t)info.sm_count * 8;
+  if (blocks > cap) blocks = cap;
+  auroc_canary_kernel<<<(unsigned)blocks, kRankThreads, 0, stream>>>(scores, labels, total, S, u2,
+                                                                     gt, eq, status);
+  cudaError_t err = cudaGetLastError();
+  if (err != cudaSuccess) return err;
+  auroc_config_kernel<<<C, kRankThreads, 0, stream>>>(labels, C, N, S, u2, auroc);
   return cudaGetLastError();
 }
 

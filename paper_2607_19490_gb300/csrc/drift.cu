@@ -156,21 +156,34 @@ drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict_
 //             (D - E^2 / (sqrt H + sqrt A)^2) / (2 sqrt(H A)), which equals
 //             (D - (sqrt H - sqrt A)^2) / (2 sqrt(H A)) without cancelling
 //             two near-equal norms.
-__global__ void drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg,
-                                      uint32_t S, uint32_t N, float *__restrict__ scores,
-                                      uint64_t stat_stride) {
-  const uint64_t seg = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (seg >= (uint64_t)S * N) return;
+// One warp per segment: lane l adds the items l, l + 32, ... in order in
+// fp64, then a fixed shuffle tree combines the lanes.
+constexpr int kFinThreads = 256;
+
+__global__ void __launch_bounds__(kFinThreads)
+drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg, uint32_t S,
+                      uint32_t N, float *__restrict__ scores, uint64_t stat_stride) {
+  const uint64_t seg = ((uint64_t)blockIdx.x * kFinThreads + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (seg >= (uint64_t)S * N) return;          // whole warps leave together
   double D = 0.0, E = 0.0, A = 0.0;
   float M = 0.f;
   const float4 *p = partials + seg * chunks_per_seg;
-  for (uint64_t c = 0; c < chunks_per_seg; ++c) {
+  for (uint64_t c = lane; c < chunks_per_seg; c += 32) {
     const float4 v = p[c];
     D += (double)v.x;
     E += (double)v.y;
     A += (double)v.z;
     M = fmaxf(M, v.w);
   }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    D += __shfl_down_sync(0xFFFFFFFFu, D, off);
+    E += __shfl_down_sync(0xFFFFFFFFu, E, off);
+    A += __shfl_down_sync(0xFFFFFFFFu, A, off);
+    M = fmaxf(M, __shfl_down_sync(0xFFFFFFFFu, M, off));
+  }
+  if (lane != 0) return;
   double rel, cosd;
   if (isnan(D) || isnan(A)) {
     rel = NAN;
@@ -195,6 +208,15 @@ __global__ void drift_finalize_kernel(const float4 *__restrict__ partials, uint6
   scores[o] = (float)rel;
   scores[stat_stride + o] = M;
   scores[2 * stat_stride + o] = (float)cosd;
+}
+
+static cudaError_t launch_finalize(const float4 *partials, uint64_t cps, uint32_t S, uint32_t N,
+                                   float *scores, uint64_t stat_stride, cudaStream_t stream) {
+  const uint64_t n_seg = (uint64_t)S * N;
+  const uint64_t blocks = (n_seg * 32 + kFinThreads - 1) / kFinThreads;
+  drift_finalize_kernel<<<(unsigned)blocks, kFinThreads, 0, stream>>>(partials, cps, S, N, scores,
+                                                                      stat_stride);
+  return cudaGetLastError();
 }
 
 // ----------------------------------------------------------------- TMA bulk pipeline
@@ -234,18 +256,16 @@ __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
-  unsigned long long state;
+  [[maybe_unused]] unsigned long long state;
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 %0, [%1], %2;"
                : "=l"(state)
                : "r"(bar), "r"(bytes)
                : "memory");
-  (void)state;
 }
 
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  unsigned long long state;
+  [[maybe_unused]] unsigned long long state;
   asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];" : "=l"(state) : "r"(bar) : "memory");
-  (void)state;
 }
 
 // true once the phase with the given parity has completed; false after
@@ -470,11 +490,7 @@ cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t 
     err = cudaGetLastError();
   }
   if (err != cudaSuccess) return err;
-  const unsigned fin_threads = 128;
-  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
-  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
-                                                                          scores, stat_stride);
-  return cudaGetLastError();
+  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
 }
 
 cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
@@ -493,11 +509,7 @@ cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, ui
                                                                      n_items, partials);
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
-  const unsigned fin_threads = 128;
-  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
-  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
-                                                                          scores, stat_stride);
-  return cudaGetLastError();
+  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
 }
 
 int drift_occupancy() {
@@ -560,11 +572,7 @@ cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32
                                                                      n_items, partials);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
-  const unsigned fin_threads = 128;
-  const uint64_t fin_blocks = (n_seg + fin_threads - 1) / fin_threads;
-  drift_finalize_kernel<<<(unsigned)fin_blocks, fin_threads, 0, stream>>>(partials, cps, S, N,
-                                                                          scores, stat_stride);
-  return cudaGetLastError();
+  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
 }
 
 }  // namespace cg
