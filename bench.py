@@ -196,9 +196,27 @@ def measured_peaks():
         return 6800.0, "fallback"
 
 
-def recorded_traffic(kernel_src: str, profile_name: str):
-    """dram bytes per launch recorded by the committed ncu summary, when the
-    kernel source still has the hash recorded there; else None."""
+KERNEL_REGIONS = {
+    # kernel -> (source file, first line of its region, text that ends the region)
+    "drift_bulk_kernel": ("drift.cu", "// ----------------------------------------------------------------- TMA bulk pipeline",
+                          "template <int NS>\nstatic cudaError_t launch_bulk"),
+    "drift_partial_kernel": ("drift.cu", "constexpr int kUnroll = 4;",
+                             "// Scores of one segment from its fp64 sums."),
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """sha256 of the source region that defines `kernel` (its device code)."""
+    fname, start, end = KERNEL_REGIONS[kernel]
+    src = open(os.path.join(ROOT, "paper_2607_19490_gb300", "csrc", fname)).read()
+    i = src.index(start)
+    j = src.index(end, i)
+    return hashlib.sha256(src[i:j].encode()).hexdigest()
+
+
+def recorded_traffic(kernel: str, profile_name: str):
+    """DRAM bytes per launch recorded by the committed ncu summary, when the
+    kernel's source region still has the hash recorded there; else None."""
     path = os.path.join(ROOT, "profiles", profile_name)
     try:
         text = open(path).read()
@@ -206,10 +224,7 @@ def recorded_traffic(kernel_src: str, profile_name: str):
         return None
     m_t = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
     m_h = re.search(r"kernel_source_sha256:\s*([0-9a-f]{64})", text)
-    if not (m_t and m_h):
-        return None
-    src = open(os.path.join(ROOT, "paper_2607_19490_gb300", "csrc", kernel_src), "rb").read()
-    if hashlib.sha256(src).hexdigest() != m_h.group(1):
+    if not (m_t and m_h) or kernel_source_hash(kernel) != m_h.group(1):
         return None
     return float(m_t.group(1))
 
@@ -387,7 +402,7 @@ def run_ours(args, ranks: Ranks):
     # whose segments are a multiple of 8 elements
     drift_kernel = ("drift_partial_kernel" if args.drift_algo == "stream" or L % 8
                     else "drift_bulk_kernel")
-    traffic = (recorded_traffic("drift.cu", f"{drift_kernel}_{args.workload}.txt")
+    traffic = (recorded_traffic(drift_kernel, f"{drift_kernel}_{args.workload}.txt")
                if args.drift_algo in ("auto", "stream", "bulk") else None)
 
     # ---- AUROC batches (configs/s): the factorial batch and a stress batch

@@ -5,13 +5,14 @@
 //   gen_setup_kernel    per-configuration draws: outlier-channel mask,
 //                       per-stage sigma (lognormal spread), flipped-channel
 //                       masks of the malicious stages; labels [N][S]
-//   gen_stats_kernel    per-segment sums the live values depend on:
+//   gen_refs_kernel     pass 1: reference normals -> fp32 references, plus
+//                       the per-chunk sums the live values depend on:
 //                       sum |a| (Eq. 2: mu = ||a||_1 / (T d)) for benign
 //                       stages under the Eq. 2 noise model; sum a^2 and
 //                       sum g^2 (the Gaussian tamper's ||v|| and ||g||)
 //   gen_coef_kernel     per-segment scalar from those sums (fixed order, fp64)
-//   gen_materialise_kernel  per 8 elements: Philox normals, reference,
-//                       benign noise or tamper, 16-byte stores
+//   gen_live_kernel     pass 2: references read back, noise or tamper
+//                       normals drawn, fp16 live values stored
 // Random draws follow the counter layout of cg_rng.cuh: element e of
 // segment seg on stream k uses block e / 4 of counter
 // (e / 4, seg, 4 config_id + k, 0).
@@ -94,16 +95,34 @@ __device__ __forceinline__ float ref_value(float z, uint32_t c, const GenParams 
   return z;
 }
 
-// ----------------------------------------------------------------- stats
-// Work item = (segment, chunk of kGenStatChunk elements).  Benign stages
-// under the Eq. 2 model sum |a|; malicious stages under the Gaussian tamper
-// sum a^2 and g^2.  Other segments write zeros.  One double2 per item.
+// ----------------------------------------------------------------- pass 1: references
+// Work item = (segment, chunk of kGenStatChunk elements).  Each thread takes
+// groups of 8 elements: two Philox blocks of reference normals, the
+// reference a (outlier channels scaled), a 16-byte store pair when the
+// group is whole and 8-aligned.  The block also reduces what the live values
+// need: sum |a| on a benign stage under the Eq. 2 model (mu = ||a||_1 / (T d));
+// sum a^2 and the tamper direction's sum g^2 on a Gaussian-tamper stage
+// (tau(v) = v + eps ||v|| g / ||g||).  One double2 per item.
+__device__ __forceinline__ void normals8(uint2 key, uint32_t q0, uint32_t seg, uint32_t c2,
+                                         uint32_t c3, int cnt, float z[8]) {
+  const float4 a = normals4(key, q0, seg, c2, c3);
+  z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
+  if (cnt > 4) {
+    const float4 b = normals4(key, q0 + 1, seg, c2, c3);
+    z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
+  } else {
+    z[4] = z[5] = z[6] = z[7] = 0.f;
+  }
+}
+
 __global__ void __launch_bounds__(kGenThreads)
-gen_stats_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
-                 double2 *__restrict__ stats) {
+gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *__restrict__ refs,
+                double2 *__restrict__ stats) {
   __shared__ double2 warp_sum[kGenThreads / 32];
   const uint64_t n_items = (uint64_t)p.S * p.N * p.stat_chunks;
   const uint2 key = philox_key(p.seed);
+  const uint32_t c2_ref = 4u * p.config_id + kStreamRef;
+  const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   const int tid = threadIdx.x;
   for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x) {
     const uint32_t seg = (uint32_t)(item / p.stat_chunks);
@@ -112,31 +131,36 @@ gen_stats_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
     const bool mal = is_malicious(p, s);
     const bool need_l1 = !mal && p.noise == CG_NOISE_PAPER;
     const bool need_l2 = mal && p.tamper == CG_TAMPER_ADDITIVE;
+    const uint64_t e_begin = ch * kGenStatChunk;
+    const uint64_t e_end = min(e_begin + (uint64_t)kGenStatChunk, p.L);
     float x = 0.f, y = 0.f;
-    if (need_l1 || need_l2) {
-      const uint64_t e_begin = ch * kGenStatChunk;
-      const uint64_t e_end = min(e_begin + (uint64_t)kGenStatChunk, p.L);
-      // blocks of 4 elements; e_begin is a multiple of 4
-      for (uint64_t q = (e_begin >> 2) + tid; 4 * q < e_end; q += kGenThreads) {
-        const float4 z = normals4(key, (uint32_t)q, seg, 4u * p.config_id + kStreamRef);
-        const float zz[4] = {z.x, z.y, z.z, z.w};
-        float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (need_l2) g = normals4(key, (uint32_t)q, seg, 4u * p.config_id + kStreamTamper);
-        const float gg[4] = {g.x, g.y, g.z, g.w};
-        uint32_t c = (uint32_t)((4 * q) % p.d);
+    for (uint64_t e0 = e_begin + 8 * (uint64_t)tid; e0 < e_end; e0 += 8 * (uint64_t)kGenThreads) {
+      const int cnt = (int)min((uint64_t)8, p.L - e0);
+      float z[8], a[8];
+      normals8(key, (uint32_t)(e0 >> 2), seg, c2_ref, 0u, cnt, z);
+      uint32_t c = (uint32_t)(e0 % p.d);
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          if (4 * q + j < e_end) {
-            const float a = ref_value(zz[j], c, p, outlier_mask);
-            if (need_l1) {
-              x += fabsf(a);
-            } else {
-              x = fmaf(a, a, x);
-              y = fmaf(gg[j], gg[j], y);
-            }
-          }
-          c = (c + 1 == p.d) ? 0 : c + 1;
+      for (int k = 0; k < 8; ++k) {
+        a[k] = ref_value(z[k], c, p, outlier_mask);
+        c = (c + 1 == p.d) ? 0 : c + 1;
+      }
+      if (need_l1) {
+        for (int k = 0; k < cnt; ++k) x += fabsf(a[k]);
+      } else if (need_l2) {
+        float g[8];
+        normals8(key, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, g);
+        for (int k = 0; k < cnt; ++k) {
+          x = fmaf(a[k], a[k], x);
+          y = fmaf(g[k], g[k], y);
         }
+      }
+      const uint64_t gidx = (uint64_t)seg * p.L + e0;
+      if (cnt == 8 && (gidx & 7) == 0) {
+        float4 *r4 = reinterpret_cast<float4 *>(refs + gidx);
+        r4[0] = make_float4(a[0], a[1], a[2], a[3]);
+        r4[1] = make_float4(a[4], a[5], a[6], a[7]);
+      } else {
+        for (int k = 0; k < cnt; ++k) refs[gidx + k] = a[k];
       }
     }
     double dx = x, dy = y;
@@ -186,17 +210,19 @@ __global__ void gen_coef_kernel(GenParams p, const double2 *__restrict__ stats,
   coef[seg] = v;
 }
 
-// ----------------------------------------------------------------- materialise
-// One thread per group of 8 segment-local elements (two Philox blocks per
-// stream).  Vector stores when the group is whole and 8-aligned globally.
+// ----------------------------------------------------------------- pass 2: live values
+// One thread per group of 8 segment-local elements: the references written
+// by pass 1 are read back (16-byte loads when the group is whole and
+// 8-aligned), the benign noise or the tamper applied, the fp16 live values
+// stored.  In recompute mode every stage is benign, its noise comes from
+// counter word 3 = the replica, and the fp16 result overwrites the
+// references in place as fp32.
 __global__ void __launch_bounds__(kGenThreads)
-gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
-                       const uint32_t *__restrict__ flip_mask, const float *__restrict__ coef,
-                       uint16_t *__restrict__ acts, float *__restrict__ refs) {
+gen_live_kernel(GenParams p, const uint32_t *__restrict__ flip_mask, const float *__restrict__ coef,
+                uint16_t *__restrict__ acts, float *__restrict__ refs) {
   const uint64_t groups_per_seg = (p.L + 7) >> 3;
   const uint64_t total = (uint64_t)p.S * p.N * groups_per_seg;
   const uint2 key = philox_key(p.seed);
-  const uint32_t c2_ref = 4u * p.config_id + kStreamRef;
   const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   for (uint64_t gi = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < total;
@@ -207,45 +233,25 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
     const uint64_t e0 = 8 * j;
     const int cnt = (int)min((uint64_t)8, p.L - e0);
     const uint32_t q0 = (uint32_t)(2 * j);
+    const uint64_t g = (uint64_t)seg * p.L + e0;
+    const bool vec = (cnt == 8) && ((g & 7) == 0);
 
-    float z[8], a[8], h[8];
-    {
-      const float4 z0 = normals4(key, q0, seg, c2_ref);
-      z[0] = z0.x; z[1] = z0.y; z[2] = z0.z; z[3] = z0.w;
-      if (cnt > 4) {
-        const float4 z1 = normals4(key, q0 + 1, seg, c2_ref);
-        z[4] = z1.x; z[5] = z1.y; z[6] = z1.z; z[7] = z1.w;
-      } else {
-        z[4] = z[5] = z[6] = z[7] = 0.f;
-      }
-    }
-    const uint32_t c0 = (uint32_t)(e0 % p.d);
-    uint32_t chan[8];
-    {
-      uint32_t c = c0;
+    float a[8], h[8];
+    if (vec) {
+      const float4 r0 = reinterpret_cast<const float4 *>(refs + g)[0];
+      const float4 r1 = reinterpret_cast<const float4 *>(refs + g)[1];
+      a[0] = r0.x; a[1] = r0.y; a[2] = r0.z; a[3] = r0.w;
+      a[4] = r1.x; a[5] = r1.y; a[6] = r1.z; a[7] = r1.w;
+    } else {
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        chan[k] = c;
-        c = (c + 1 == p.d) ? 0 : c + 1;
-      }
+      for (int k = 0; k < 8; ++k) a[k] = (k < cnt) ? refs[g + k] : 0.f;
     }
-#pragma unroll
-    for (int k = 0; k < 8; ++k) a[k] = ref_value(z[k], chan[k], p, outlier_mask);
 
     const bool mal = is_malicious(p, s);
     const float cf = coef[seg];
     if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
-      const uint32_t c2 = mal ? c2_tamper : c2_noise;
-      const uint32_t c3 = mal ? 0u : p.noise_c3;
       float n[8];
-      const float4 n0 = normals4(key, q0, seg, c2, c3);
-      n[0] = n0.x; n[1] = n0.y; n[2] = n0.z; n[3] = n0.w;
-      if (cnt > 4) {
-        const float4 n1 = normals4(key, q0 + 1, seg, c2, c3);
-        n[4] = n1.x; n[5] = n1.y; n[6] = n1.z; n[7] = n1.w;
-      } else {
-        n[4] = n[5] = n[6] = n[7] = 0.f;
-      }
+      normals8(key, q0, seg, mal ? c2_tamper : c2_noise, mal ? 0u : p.noise_c3, cnt, n);
       if (!mal && p.noise == CG_NOISE_MULT) {
 #pragma unroll
         for (int k = 0; k < 8; ++k) h[k] = a[k] * (1.0f + cf * n[k]);   // a (1 + sigma_s z)
@@ -255,8 +261,12 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
       }
     } else if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS) {
       const uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
+      uint32_t c = (uint32_t)(e0 % p.d);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) h[k] = mask_bit(row, chan[k]) ? -a[k] : a[k];
+      for (int k = 0; k < 8; ++k) {
+        h[k] = mask_bit(row, c) ? -a[k] : a[k];
+        c = (c + 1 == p.d) ? 0 : c + 1;
+      }
     } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
 #pragma unroll
       for (int k = 0; k < 8; ++k) h[k] = -a[k];
@@ -265,14 +275,13 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
       for (int k = 0; k < 8; ++k) h[k] = cf * a[k];
     }
 
-    const uint64_t g = (uint64_t)seg * p.L + e0;
     if (p.recompute) {
-      // independent benign recompute: the fp16 output, stored as fp32
-      if (cnt == 8 && (g & 7) == 0) {
-        float4 *r4 = reinterpret_cast<float4 *>(refs + g);
+      // independent benign recompute: the fp16 output, stored as fp32 in place
+      if (vec) {
         float v[8];
 #pragma unroll
         for (int k = 0; k < 8; ++k) v[k] = __half2float(__float2half_rn(h[k]));
+        float4 *r4 = reinterpret_cast<float4 *>(refs + g);
         r4[0] = make_float4(v[0], v[1], v[2], v[3]);
         r4[1] = make_float4(v[4], v[5], v[6], v[7]);
       } else {
@@ -280,10 +289,7 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
       }
       continue;
     }
-    if (cnt == 8 && (g & 7) == 0) {
-      float4 *r4 = reinterpret_cast<float4 *>(refs + g);
-      r4[0] = make_float4(a[0], a[1], a[2], a[3]);
-      r4[1] = make_float4(a[4], a[5], a[6], a[7]);
+    if (vec) {
       uint4 hv;
       hv.x = (uint32_t)__half_as_ushort(__float2half_rn(h[0])) |
              ((uint32_t)__half_as_ushort(__float2half_rn(h[1])) << 16);
@@ -295,10 +301,7 @@ gen_materialise_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
              ((uint32_t)__half_as_ushort(__float2half_rn(h[7])) << 16);
       *reinterpret_cast<uint4 *>(acts + g) = hv;
     } else {
-      for (int k = 0; k < cnt; ++k) {
-        refs[g + k] = a[k];
-        acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
-      }
+      for (int k = 0; k < cnt; ++k) acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
     }
   }
 }
@@ -373,27 +376,18 @@ cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
 
   const uint64_t n_seg = (uint64_t)p.S * p.N;
-  const bool any_stats = (p.noise == CG_NOISE_PAPER) || (p.tamper == CG_TAMPER_ADDITIVE);
   const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)info.gen_blocks_per_sm;
-  if (any_stats) {
-    const uint64_t n_items = n_seg * p.stat_chunks;
-    const uint64_t grid = n_items < resident ? n_items : resident;
-    gen_stats_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, outlier_mask, stats);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  } else {
-    if ((err = cudaMemsetAsync(stats, 0, (size_t)n_seg * p.stat_chunks * 16, stream)) !=
-        cudaSuccess)
-      return err;
-  }
+  const uint64_t n_items = n_seg * p.stat_chunks;
+  const uint64_t grid1 = n_items < resident ? n_items : resident;
+  gen_refs_kernel<<<(unsigned)grid1, kGenThreads, 0, stream>>>(p, outlier_mask, refs, stats);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
   gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, stats, stage_sigma, coef);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
 
   const uint64_t groups = n_seg * ((p.L + 7) >> 3);
   const uint64_t blocks_needed = (groups + kGenThreads - 1) / kGenThreads;
   const uint64_t grid = blocks_needed < resident * 4 ? blocks_needed : resident * 4;
-  gen_materialise_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, outlier_mask, flip_mask,
-                                                                     coef, acts, refs);
-  // (in recompute mode acts is unused and refs receives the recompute)
+  gen_live_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, flip_mask, coef, acts, refs);
   return cudaGetLastError();
 }
 
@@ -421,7 +415,7 @@ cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint3
 
 int gen_occupancy() {
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_materialise_kernel, kGenThreads, 0) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_live_kernel, kGenThreads, 0) !=
       cudaSuccess)
     return 0;
   return n;
