@@ -520,6 +520,105 @@ int or_generate_pipeline(const or_desc *D, uint16_t *acts, float *refs,
   return err;
 }
 
+/* Propagating pipeline (Eq. 2's recursion h_i = f_i(h_{i-1}) + delta_i     */
+/* with the block's response to its input linearised as                     */
+/*     f_i(h_{i-1}) = a_i + gain * (h_{i-1} - a_{i-1}),                     */
+/* h_{-1} = a_{-1}, i.e. the first stage sees the exact embedding).  With   */
+/* v_i = f_i(h_{i-1}):                                                       */
+/*   benign    h_i = fp16(v_i + sigma_i mu_i z), mu_i = ||v_i||_1 / (T d)    */
+/*             (MULT: fp16(v_i (1 + sigma_i z)))                            */
+/*   malicious h_i = fp16(tau(v_i)) (Eq. 3 with v = f(h_{i*-1}), Sec. 3.2)   */
+/* Stages are produced in order, each from the previous stage's fp16 live   */
+/* values; gain = 0 is the hop-local pipeline of or_generate_pipeline.      */
+int or_generate_propagating(const or_desc *D, double gain, uint16_t *acts,
+                            float *refs, int n_threads) {
+  int st = check_desc(D);
+  if (st) return st;
+  or_tables t;
+  st = build_tables(D, &t);
+  if (st) return st;
+  const uint32_t S = D->n_shards, N = D->n_canaries, d = D->hidden;
+  const uint64_t L = (uint64_t)D->tokens * d;
+  int err = OR_OK;
+#ifdef _OPENMP
+  if (n_threads > 0) omp_set_num_threads(n_threads);
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+  for (int64_t nn = 0; nn < (int64_t)N; ++nn) {
+    const uint32_t n = (uint32_t)nn;
+    uint32_t key[2];
+    seed_to_key(D->seed, key);
+    double *a = (double *)malloc(L * sizeof(double));
+    double *v = (double *)malloc(L * sizeof(double));
+    double *dev = (double *)calloc(L, sizeof(double));   /* h_{i-1} - a_{i-1} */
+    if (!a || !v || !dev) {
+      free(a); free(v); free(dev);
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+      err = OR_NO_MEMORY;
+      continue;
+    }
+    for (uint32_t s = 0; s < S; ++s) {
+      const uint32_t seg = s * N + n;
+      const size_t off = (size_t)seg * L;
+      for (uint64_t e = 0; e < L; ++e) {
+        uint32_t c = (uint32_t)(e % d);
+        double scale = 1.0;
+        for (uint32_t j = 0; j < D->n_outlier; ++j)
+          if (t.outlier[j] == c) scale = D->outlier_scale;
+        float af = (float)(element_normal(key, seg, D->config_id, OR_STREAM_REF, e) * scale);
+        a[e] = (double)af;
+        if (refs) refs[off + e] = af;
+        v[e] = a[e] + gain * dev[e];
+      }
+      double *live = dev;   /* reuse: live values of this stage */
+      if (!t.is_mal[s]) {
+        double sig = t.shard_sigma[s];
+        if (D->noise == OR_NOISE_MULT) {
+          for (uint64_t e = 0; e < L; ++e)
+            live[e] = v[e] * (1.0 + sig * element_normal(key, seg, D->config_id,
+                                                          OR_STREAM_NOISE, e));
+        } else {
+          double l1 = 0.0;
+          for (uint64_t e = 0; e < L; ++e) l1 += fabs(v[e]);
+          double coef = sig * (l1 / (double)L);
+          for (uint64_t e = 0; e < L; ++e)
+            live[e] = v[e] + coef * element_normal(key, seg, D->config_id,
+                                                   OR_STREAM_NOISE, e);
+        }
+      } else if (D->tamper == OR_TAMPER_ADDITIVE) {
+        double vv = 0.0, gg = 0.0;
+        for (uint64_t e = 0; e < L; ++e) {
+          double g = element_normal(key, seg, D->config_id, OR_STREAM_TAMPER, e);
+          vv += v[e] * v[e];
+          gg += g * g;
+        }
+        double coef = (gg > 0.0) ? D->tamper_param * sqrt(vv) / sqrt(gg) : 0.0;
+        for (uint64_t e = 0; e < L; ++e)
+          live[e] = v[e] + coef * element_normal(key, seg, D->config_id,
+                                                 OR_STREAM_TAMPER, e);
+      } else if (D->tamper == OR_TAMPER_SIGNFLIP_CHANNELS) {
+        for (uint64_t e = 0; e < L; ++e)
+          live[e] = t.flip[(size_t)s * d + (uint32_t)(e % d)] ? -v[e] : v[e];
+      } else if (D->tamper == OR_TAMPER_SIGNFLIP_FULL) {
+        for (uint64_t e = 0; e < L; ++e) live[e] = -v[e];
+      } else {
+        for (uint64_t e = 0; e < L; ++e) live[e] = D->tamper_param * v[e];
+      }
+      for (uint64_t e = 0; e < L; ++e) {
+        uint16_t hb = or_half_from_double(live[e]);
+        if (acts) acts[off + e] = hb;
+        dev[e] = or_half_to_double(hb) - a[e];
+      }
+    }
+    free(a); free(v); free(dev);
+  }
+  free_tables(&t);
+  (void)n_threads;
+  return err;
+}
+
 /* An independent benign recompute of every stage (Sec. 4.5, redundant-     */
 /* recompute ceiling; Sec. 4.4, noisy reference): the benign output of each */
 /* stage, malicious ones included, with the noise of replica r, rounded to  */

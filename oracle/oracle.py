@@ -111,6 +111,9 @@ def lib():
                                           P(ctypes.c_int64), P(ctypes.c_int64), P(ctypes.c_int64),
                                           P(dbl)]
             L.or_auroc_pooled.restype = i32
+            L.or_generate_propagating.argtypes = [P(_Desc), dbl, P(ctypes.c_uint16), P(ctypes.c_float),
+                                                  ctypes.c_int]
+            L.or_generate_propagating.restype = i32
         return _lib
 
 
@@ -229,6 +232,17 @@ def generate_pipeline(desc, n_threads=0):
                                       _p(refs, ctypes.c_float), _p(labels, ctypes.c_int8),
                                       int(n_threads)))
     return acts, refs, labels
+
+
+def generate_propagating(desc, gain, n_threads=0):
+    """Pipeline whose stages inherit the upstream deviation with `gain`
+    (binary32 value): acts uint16 and refs float32 [S][N][T*d]."""
+    S, N, L = desc.n_shards, desc.n_canaries, desc.tokens * desc.hidden
+    acts = np.zeros((S, N, L), dtype=np.uint16)
+    refs = np.zeros((S, N, L), dtype=np.float32)
+    _check(lib().or_generate_propagating(ctypes.byref(desc), _f32(gain), _p(acts, ctypes.c_uint16),
+                                         _p(refs, ctypes.c_float), int(n_threads)))
+    return acts, refs
 
 
 def generate_recompute(desc, replica, n_threads=0):
