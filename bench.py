@@ -575,7 +575,12 @@ def study_pass(cg, torch, configs, dev, bufs, res):
         refs = bufs["refs"][:E].view(S, N, L)
         labels = bufs["labels"][:N * S].view(1, N, S)
         ctrl = bufs["ctrl"][:N * S].view(1, N, S)
-        cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"], status=bufs["status"])
+        if cfg.get("gain", 0.0):
+            cg.cg_generate_propagating(desc, cfg["gain"], acts, refs, labels[0], bufs["gws"],
+                                       status=bufs["status"])
+        else:
+            cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"],
+                                    status=bufs["status"])
         scores = bufs["scores"][:3 * N * S].view(3, N, S)
         cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"], status=bufs["status"])
         cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
@@ -665,10 +670,19 @@ def run_study(args, ranks: Ranks):
         "auroc_summary": summary,
         "per_config_auroc": {n: [round(float(x), 6) for x in A[:, k]] for k, n in enumerate(names)},
         "cpu_baseline": cpu,
-        "gpu_launches": 12 * len(configs) * reps,
+        "gpu_launches": sum(launches_per_config(c) for c in configs) * reps,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
+
+
+def launches_per_config(cfg) -> int:
+    """Kernel launches of one study configuration: generator (4, or 2 + 3 per
+    stage when propagating), drift scores (2), control labels (1), three
+    per-canary AUROC calls and the control's (2 launches each for a single
+    configuration), pooled AUROC (1)."""
+    gen = 2 + 3 * cfg["n_shards"] if cfg.get("gain", 0.0) else 4
+    return gen + 2 + 1 + 4 * 2 + 1
 
 
 def study_oracle_baseline(configs, seconds):
@@ -680,8 +694,11 @@ def study_oracle_baseline(configs, seconds):
     done, t0 = 0, time.perf_counter()
     for cfg in configs:
         sub = SI.shrink(cfg, n_canaries=min(8, cfg["n_canaries"]))
+        gain = sub.pop("gain", 0.0)
         D = O.desc_from_dict(sub)
         acts, refs, labels = O.generate_pipeline(D, n_threads=threads)
+        if gain:
+            acts, refs = O.generate_propagating(D, gain, n_threads=threads)
         sc = O.drift_scores(acts, refs, sub["n_shards"], sub["n_canaries"], n_threads=threads)
         for k in range(3):
             O.auroc(sc[k].astype(np.float32)[None], labels[None])

@@ -166,6 +166,21 @@ cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica,
                                 int32_t *d_status, cg_stream_t stream);
 
 /*
+ * A pipeline whose stages inherit the upstream deviation (Eq. 2's recursion
+ * h_i = f_i(h_{i-1}) + delta_i), with each block's response to its input
+ * linearised as f_i(h_{i-1}) = a_i + gain (h_{i-1} - a_{i-1}); the first
+ * stage sees the exact embedding.  Benign stages add Eq. 2 noise to
+ * v_i = f_i(h_{i-1}) (mu_i = ||v_i||_1 / (T d)); malicious stages output
+ * fp16(tau(v_i)) (Eq. 3).  gain = 0 gives cg_generate_pipeline's output.
+ * Arguments, layouts and workspace as cg_generate_pipeline; the stages are
+ * produced in order (3 launches per stage).
+ */
+cg_status cg_generate_propagating(const cg_pipeline_desc *desc, float gain,
+                                  uint16_t *d_acts, float *d_refs, int8_t *d_labels,
+                                  void *d_ws, size_t ws_bytes, int32_t *d_status,
+                                  cg_stream_t stream);
+
+/*
  * Random-baseline scores (Sec. 4.5): d_scores[c][n][s] ~ Uniform(0, 1),
  * the top 24 bits of word s of Philox aux stream 5 (canary n, config id
  * config_id0 + c) times 2^-24.  fp32 [C][N][S], 4-byte aligned.

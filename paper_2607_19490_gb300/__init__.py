@@ -22,7 +22,7 @@ __all__ = [
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
     "cg_drift_scores_ex", "cg_drift_scores_host", "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
-    "cg_random_scores", "cg_auroc_pooled",
+    "cg_random_scores", "cg_auroc_pooled", "cg_generate_propagating",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
     "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
 ]
@@ -97,6 +97,7 @@ def load() -> ctypes.CDLL:
             "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
             "cg_generate_recompute": ([ctypes.POINTER(PipelineDesc), u32, P, P, sz, P, P], ctypes.c_int),
+            "cg_generate_propagating": ([ctypes.POINTER(PipelineDesc), ctypes.c_float, P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_random_scores": ([u64, u32, u32, u32, u32, P, P], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_ex": ([P, P, u32, u32, u64, P, u64, P, sz, P, ctypes.c_int32, P], ctypes.c_int),
@@ -239,6 +240,30 @@ def cg_generate_recompute(desc: PipelineDesc, replica, out=None, ws=None, status
                                         ws.numel(), _ptr(status), _stream(stream)),
            "cg_generate_recompute")
     return out
+
+
+def cg_generate_propagating(desc: PipelineDesc, gain, acts=None, refs=None, labels=None, ws=None,
+                            status=None, stream=None):
+    """Pipeline whose stages inherit gain x the upstream deviation; returns
+    (acts fp16, refs fp32, labels int8) like cg_generate_pipeline."""
+    torch = _torch()
+    S, N, L = desc.n_shards, desc.n_canaries, desc.seg_len
+    acts = torch.empty((S, N, L), dtype=torch.float16, device="cuda") if acts is None else acts
+    refs = torch.empty((S, N, L), dtype=torch.float32, device="cuda") if refs is None else refs
+    labels = torch.empty((N, S), dtype=torch.int8, device="cuda") if labels is None else labels
+    ws = (torch.empty(cg_generate_workspace_size(desc), dtype=torch.uint8, device="cuda")
+          if ws is None else ws)
+    _cuda(acts, "acts", (torch.float16,))
+    _cuda(refs, "refs", (torch.float32,))
+    _cuda(labels, "labels", (torch.int8,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    if acts.numel() != S * N * L or refs.numel() != S * N * L or labels.numel() != N * S:
+        raise ValueError("acts/refs must hold S*N*T*d elements and labels N*S")
+    _check(load().cg_generate_propagating(ctypes.byref(desc), float(gain), _ptr(acts), _ptr(refs),
+                                          _ptr(labels), _ptr(ws), ws.numel(), _ptr(status),
+                                          _stream(stream)), "cg_generate_propagating")
+    return acts, refs, labels
 
 
 def cg_random_scores(seed, n_configs, n_canaries, n_shards, config_id0=0, out=None, stream=None):

@@ -199,6 +199,23 @@ cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica, 
                                        (cudaStream_t)stream));
 }
 
+cg_status cg_generate_propagating(const cg_pipeline_desc *desc, float gain, uint16_t *d_acts,
+                                  float *d_refs, int8_t *d_labels, void *d_ws, size_t ws_bytes,
+                                  int32_t *d_status, cg_stream_t stream) {
+  cg_status st = check_desc(desc);
+  if (st != CG_OK) return st;
+  if (!isfinite(gain)) return CG_ERR_INVALID_ARG;
+  if (!d_acts || !d_refs) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  const cg::GenLayout lay = cg::gen_layout(*desc);
+  if (!d_ws || ws_bytes < lay.total) return CG_ERR_WORKSPACE;
+  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
+  cg::GenParams p = make_params(*desc, lay);
+  return from_cuda(cg::launch_generate_propagating(p, gain, d_acts, d_refs, d_labels, d_ws, lay,
+                                                   d_status, (cudaStream_t)stream));
+}
+
 cg_status cg_random_scores(uint64_t seed, uint32_t config_id0, uint32_t n_configs,
                            uint32_t n_canaries, uint32_t n_shards, float *d_scores,
                            cg_stream_t stream) {

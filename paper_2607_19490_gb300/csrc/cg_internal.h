@@ -81,6 +81,9 @@ struct GenParams {
 cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int8_t *labels,
                             void *ws, const GenLayout &lay, int32_t *status, cudaStream_t stream);
 
+cudaError_t launch_generate_propagating(const GenParams &p, float gain, uint16_t *acts, float *refs,
+                                       int8_t *labels, void *ws, const GenLayout &lay,
+                                       int32_t *status, cudaStream_t stream);
 cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
                                  uint32_t S, float *out, cudaStream_t stream);
 

@@ -306,6 +306,179 @@ gen_live_kernel(GenParams p, const uint32_t *__restrict__ flip_mask, const float
   }
 }
 
+// ----------------------------------------------------------------- propagating pipeline
+// Eq. 2's recursion with the block's response to its input linearised:
+//   v_s = f_s(h_{s-1}) = a_s + gain (h_{s-1} - a_{s-1}),  v_0 = a_0,
+// benign h_s = fp16(v_s + sigma_s mu_s z) (mu_s = ||v_s||_1 / (T d)) or
+// fp16(v_s (1 + sigma_s z)); malicious h_s = fp16(tau(v_s)).  Stage s reads
+// stage s-1's stored fp16 live values and fp32 references, so the stages
+// run one after the other.
+__device__ __forceinline__ void prop_inputs(const GenParams &p, uint32_t s, float gain,
+                                            const float *refs, const uint16_t *acts, uint64_t g,
+                                            uint64_t gprev, int cnt, bool vec, float v[8]) {
+  float a[8], ap[8], hp[8];
+  if (vec) {
+    const float4 r0 = reinterpret_cast<const float4 *>(refs + g)[0];
+    const float4 r1 = reinterpret_cast<const float4 *>(refs + g)[1];
+    a[0] = r0.x; a[1] = r0.y; a[2] = r0.z; a[3] = r0.w;
+    a[4] = r1.x; a[5] = r1.y; a[6] = r1.z; a[7] = r1.w;
+  } else {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) a[k] = (k < cnt) ? refs[g + k] : 0.f;
+  }
+  if (s == 0) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = a[k];
+    return;
+  }
+  if (vec) {
+    const float4 r0 = reinterpret_cast<const float4 *>(refs + gprev)[0];
+    const float4 r1 = reinterpret_cast<const float4 *>(refs + gprev)[1];
+    ap[0] = r0.x; ap[1] = r0.y; ap[2] = r0.z; ap[3] = r0.w;
+    ap[4] = r1.x; ap[5] = r1.y; ap[6] = r1.z; ap[7] = r1.w;
+    const uint4 hv = *reinterpret_cast<const uint4 *>(acts + gprev);
+    const uint32_t w[4] = {hv.x, hv.y, hv.z, hv.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      hp[2 * k] = __half2float(__ushort_as_half((uint16_t)(w[k] & 0xFFFFu)));
+      hp[2 * k + 1] = __half2float(__ushort_as_half((uint16_t)(w[k] >> 16)));
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      ap[k] = (k < cnt) ? refs[gprev + k] : 0.f;
+      hp[k] = (k < cnt) ? __half2float(__ushort_as_half(acts[gprev + k])) : 0.f;
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) v[k] = fmaf(gain, hp[k] - ap[k], a[k]);
+}
+
+__global__ void __launch_bounds__(kGenThreads)
+gen_prop_stats_kernel(GenParams p, uint32_t s, float gain, const float *__restrict__ refs,
+                      const uint16_t *__restrict__ acts, double2 *__restrict__ stats) {
+  __shared__ double2 warp_sum[kGenThreads / 32];
+  const uint64_t n_items = (uint64_t)p.N * p.stat_chunks;
+  const uint2 key = philox_key(p.seed);
+  const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
+  const bool mal = is_malicious(p, s);
+  const bool need_l1 = !mal && p.noise == CG_NOISE_PAPER;
+  const bool need_l2 = mal && p.tamper == CG_TAMPER_ADDITIVE;
+  const int tid = threadIdx.x;
+  for (uint64_t it = blockIdx.x; it < n_items; it += gridDim.x) {
+    const uint32_t n = (uint32_t)(it / p.stat_chunks);
+    const uint64_t ch = it - (uint64_t)n * p.stat_chunks;
+    const uint32_t seg = s * p.N + n;
+    const uint64_t e_begin = ch * kGenStatChunk;
+    const uint64_t e_end = min(e_begin + (uint64_t)kGenStatChunk, p.L);
+    float x = 0.f, y = 0.f;
+    if (need_l1 || need_l2) {
+      for (uint64_t e0 = e_begin + 8 * (uint64_t)tid; e0 < e_end;
+           e0 += 8 * (uint64_t)kGenThreads) {
+        const int cnt = (int)min((uint64_t)8, p.L - e0);
+        const uint64_t g = (uint64_t)seg * p.L + e0;
+        const uint64_t gprev = g - (s ? (uint64_t)p.N * p.L : 0);
+        const bool vec = (cnt == 8) && ((g & 7) == 0) && ((gprev & 7) == 0);
+        float v[8];
+        prop_inputs(p, s, gain, refs, acts, g, gprev, cnt, vec, v);
+        if (need_l1) {
+          for (int k = 0; k < cnt; ++k) x += fabsf(v[k]);
+        } else {
+          float gg[8];
+          normals8(key, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, gg);
+          for (int k = 0; k < cnt; ++k) {
+            x = fmaf(v[k], v[k], x);
+            y = fmaf(gg[k], gg[k], y);
+          }
+        }
+      }
+    }
+    double dx = x, dy = y;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      dx += __shfl_down_sync(0xFFFFFFFFu, dx, off);
+      dy += __shfl_down_sync(0xFFFFFFFFu, dy, off);
+    }
+    if ((tid & 31) == 0) warp_sum[tid >> 5] = make_double2(dx, dy);
+    __syncthreads();
+    if (tid == 0) {
+      double2 t = make_double2(0.0, 0.0);
+      for (int w = 0; w < kGenThreads / 32; ++w) {
+        t.x += warp_sum[w].x;
+        t.y += warp_sum[w].y;
+      }
+      stats[(uint64_t)seg * p.stat_chunks + ch] = t;
+    }
+    __syncthreads();
+  }
+}
+
+__global__ void __launch_bounds__(kGenThreads)
+gen_prop_live_kernel(GenParams p, uint32_t s, float gain, const uint32_t *__restrict__ flip_mask,
+                     const float *__restrict__ coef, const float *__restrict__ refs,
+                     uint16_t *__restrict__ acts) {
+  const uint64_t groups_per_seg = (p.L + 7) >> 3;
+  const uint64_t total = (uint64_t)p.N * groups_per_seg;
+  const uint2 key = philox_key(p.seed);
+  const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
+  const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
+  const bool mal = is_malicious(p, s);
+  for (uint64_t gi = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < total;
+       gi += (uint64_t)gridDim.x * blockDim.x) {
+    const uint32_t n = (uint32_t)(gi / groups_per_seg);
+    const uint64_t j = gi - (uint64_t)n * groups_per_seg;
+    const uint32_t seg = s * p.N + n;
+    const uint64_t e0 = 8 * j;
+    const int cnt = (int)min((uint64_t)8, p.L - e0);
+    const uint32_t q0 = (uint32_t)(2 * j);
+    const uint64_t g = (uint64_t)seg * p.L + e0;
+    const uint64_t gprev = g - (s ? (uint64_t)p.N * p.L : 0);
+    const bool vec = (cnt == 8) && ((g & 7) == 0) && ((gprev & 7) == 0);
+    float v[8], h[8];
+    prop_inputs(p, s, gain, refs, acts, g, gprev, cnt, vec, v);
+    const float cf = coef[seg];
+    if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
+      float z[8];
+      normals8(key, q0, seg, mal ? c2_tamper : c2_noise, 0u, cnt, z);
+      if (!mal && p.noise == CG_NOISE_MULT) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[k] = v[k] * (1.0f + cf * z[k]);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) h[k] = fmaf(cf, z[k], v[k]);
+      }
+    } else if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS) {
+      const uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
+      uint32_t c = (uint32_t)(e0 % p.d);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        h[k] = mask_bit(row, c) ? -v[k] : v[k];
+        c = (c + 1 == p.d) ? 0 : c + 1;
+      }
+    } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = -v[k];
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = cf * v[k];
+    }
+    if (vec) {
+      uint4 hv;
+      hv.x = (uint32_t)__half_as_ushort(__float2half_rn(h[0])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[1])) << 16);
+      hv.y = (uint32_t)__half_as_ushort(__float2half_rn(h[2])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[3])) << 16);
+      hv.z = (uint32_t)__half_as_ushort(__float2half_rn(h[4])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[5])) << 16);
+      hv.w = (uint32_t)__half_as_ushort(__float2half_rn(h[6])) |
+             ((uint32_t)__half_as_ushort(__float2half_rn(h[7])) << 16);
+      *reinterpret_cast<uint4 *>(acts + g) = hv;
+    } else {
+      for (int k = 0; k < cnt; ++k) acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
+    }
+  }
+}
+
 // ----------------------------------------------------------------- random baseline
 // Sec. 4.5: every score replaced by Uniform(0, 1).  Thread per (config,
 // canary); score s = (x >> 8) 2^-24 with x word s of aux stream
@@ -389,6 +562,44 @@ cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int
   const uint64_t grid = blocks_needed < resident * 4 ? blocks_needed : resident * 4;
   gen_live_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, flip_mask, coef, acts, refs);
   return cudaGetLastError();
+}
+
+cudaError_t launch_generate_propagating(const GenParams &p, float gain, uint16_t *acts, float *refs,
+                                       int8_t *labels, void *ws, const GenLayout &lay,
+                                       int32_t *status, cudaStream_t stream) {
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  char *base = static_cast<char *>(ws);
+  uint32_t *outlier_mask = reinterpret_cast<uint32_t *>(base + lay.outlier_mask);
+  uint32_t *flip_mask = reinterpret_cast<uint32_t *>(base + lay.flip_mask);
+  float *stage_sigma = reinterpret_cast<float *>(base + lay.stage_sigma);
+  float *coef = reinterpret_cast<float *>(base + lay.seg_coef);
+  double2 *stats = reinterpret_cast<double2 *>(base + lay.stats);
+  cudaError_t err;
+  gen_setup_kernel<<<1, 256, 0, stream>>>(p, outlier_mask, flip_mask, stage_sigma, labels, status);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const uint64_t n_seg = (uint64_t)p.S * p.N;
+  const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)info.gen_blocks_per_sm;
+  // every stage's reference first (its statistics are recomputed below)
+  const uint64_t n_items = n_seg * p.stat_chunks;
+  gen_refs_kernel<<<(unsigned)(n_items < resident ? n_items : resident), kGenThreads, 0, stream>>>(
+      p, outlier_mask, refs, stats);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const uint64_t stage_items = (uint64_t)p.N * p.stat_chunks;
+  const uint64_t stage_groups = (uint64_t)p.N * ((p.L + 7) >> 3);
+  const uint64_t live_blocks = (stage_groups + kGenThreads - 1) / kGenThreads;
+  for (uint32_t s = 0; s < p.S; ++s) {
+    gen_prop_stats_kernel<<<(unsigned)(stage_items < resident ? stage_items : resident), kGenThreads,
+                            0, stream>>>(p, s, gain, refs, acts, stats);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, stats, stage_sigma,
+                                                                         coef);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    gen_prop_live_kernel<<<(unsigned)(live_blocks < resident * 4 ? live_blocks : resident * 4),
+                           kGenThreads, 0, stream>>>(p, s, gain, flip_mask, coef, refs, acts);
+    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,

@@ -248,3 +248,20 @@ STUDIES = {
     "depth": depth_configs,
     "paper_snr": paper_snr_configs,
 }
+
+
+PROPAGATION_GAINS = (0.0, 0.5, 0.9, 1.0, 1.2)
+
+
+def propagation_configs(seeds=SUBSTUDY_SEEDS):
+    """Deviations that propagate along the pipeline (Eq. 2's recursion with a
+    linearised block gain): gain x {first, middle, last} attacker position."""
+    out = []
+    for j, gain in enumerate(PROPAGATION_GAINS):
+        for p, pos in enumerate((0, 5, 11)):
+            out += [dict(anchor(malicious=(pos,), seed=sd, config_id=600 + 30 * j + 10 * p + i),
+                         gain=gain) for i, sd in enumerate(seeds)]
+    return out
+
+
+STUDIES["propagation"] = propagation_configs
