@@ -153,6 +153,153 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
   }
 }
 
+// Grouped ranking for S <= 32: G = the next power of two >= S lanes per
+// canary, so one warp ranks 32 / G canaries at once; the shuffles run
+// within each G-lane group (width G).  Lane j of a group holds stage j.
+template <int G>
+__device__ __forceinline__ void group_counts(const float *__restrict__ scores,
+                                             const int8_t *__restrict__ labels, uint64_t o,
+                                             bool active, uint32_t S, int lane, long long &g,
+                                             long long &e, int &nm, int &nb, bool &saw_nan) {
+  const int sub = lane & (G - 1);
+  const bool in = active && (uint32_t)sub < S;
+  const float m = in ? scores[o * S + sub] : 0.f;
+  const int l = in ? (int)labels[o * S + sub] : -1;
+  if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
+  int lg = 0, le = 0;
+  for (uint32_t k = 0; k < S; ++k) {
+    const float mk = __shfl_sync(0xFFFFFFFFu, m, (int)k, G);
+    const int lk = __shfl_sync(0xFFFFFFFFu, l, (int)k, G);
+    if (l == 1 && lk == 0) {
+      lg += (m > mk);
+      le += (m == mk);
+    }
+  }
+  const unsigned shift = (unsigned)(lane & ~(G - 1));
+  const unsigned gmask = (G == 32) ? 0xFFFFFFFFu : ((1u << G) - 1u);
+  nm = __popc((__ballot_sync(0xFFFFFFFFu, l == 1) >> shift) & gmask);
+  nb = __popc((__ballot_sync(0xFFFFFFFFu, l == 0) >> shift) & gmask);
+#pragma unroll
+  for (int off = G / 2; off > 0; off >>= 1) {
+    lg += __shfl_xor_sync(0xFFFFFFFFu, lg, off, G);
+    le += __shfl_xor_sync(0xFFFFFFFFu, le, off, G);
+  }
+  g = lg;
+  e = le;
+}
+
+// One block per configuration (many configurations).
+template <int G>
+__global__ void __launch_bounds__(kRankThreads)
+auroc_grouped_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                     uint32_t C, uint32_t N, uint32_t S, int64_t *__restrict__ u2_out,
+                     int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
+                     double *__restrict__ auroc, int32_t *status) {
+  constexpr int kPerWarp = 32 / G;
+  __shared__ long long red[kRankWarps][4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const bool leader = (lane & (G - 1)) == 0;
+  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
+    long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
+    bool saw_nan = false;
+    for (uint32_t n0 = (uint32_t)warp * kPerWarp; n0 < N; n0 += kRankWarps * kPerWarp) {
+      const uint32_t n = n0 + (uint32_t)(lane / G);
+      const bool active = n < N;
+      const uint64_t o = (uint64_t)c * N + n;
+      long long g, e;
+      int nm, nb;
+      group_counts<G>(scores, labels, o, active, S, lane, g, e, nm, nb, saw_nan);
+      if (leader && active) {
+        const long long u2 = 2 * g + e;
+        u2_out[o] = u2;
+        if (gt_out) gt_out[o] = g;
+        if (eq_out) eq_out[o] = e;
+        const long long pairs = (long long)nm * nb;
+        if (pairs > 0) {
+          total += u2;
+          valid += 1;
+          pmin = min(pmin, pairs);
+          pmax = max(pmax, pairs);
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      total += __shfl_down_sync(0xFFFFFFFFu, total, off);
+      valid += __shfl_down_sync(0xFFFFFFFFu, valid, off);
+      pmin = min(pmin, __shfl_down_sync(0xFFFFFFFFu, pmin, off));
+      pmax = max(pmax, __shfl_down_sync(0xFFFFFFFFu, pmax, off));
+    }
+    if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
+      atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+    if (lane == 0) {
+      red[warp][0] = total;
+      red[warp][1] = valid;
+      red[warp][2] = pmin;
+      red[warp][3] = pmax;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < kRankWarps; ++w) {
+        red[0][0] += red[w][0];
+        red[0][1] += red[w][1];
+        red[0][2] = min(red[0][2], red[w][2]);
+        red[0][3] = max(red[0][3], red[w][3]);
+      }
+      const long long T = red[0][0], V = red[0][1];
+      double A;
+      if (V == 0) {
+        A = NAN;
+      } else if (red[0][2] == red[0][3]) {
+        A = __ddiv_rn((double)T, (double)(2 * red[0][2] * V));
+      } else {
+        double acc = 0.0;
+        for (uint32_t n = 0; n < N; ++n) {
+          const int8_t *l = labels + ((uint64_t)c * N + n) * S;
+          long long nm = 0, nb = 0;
+          for (uint32_t s = 0; s < S; ++s) {
+            nm += (l[s] == 1);
+            nb += (l[s] == 0);
+          }
+          if (nm * nb == 0) continue;
+          acc = __dadd_rn(acc, __ddiv_rn((double)u2_out[(uint64_t)c * N + n], (double)(2 * nm * nb)));
+        }
+        A = __ddiv_rn(acc, (double)V);
+      }
+      auroc[c] = A;
+    }
+    __syncthreads();
+  }
+}
+
+// Canary-parallel counts for few configurations (combine: auroc_config_kernel).
+template <int G>
+__global__ void __launch_bounds__(kRankThreads)
+auroc_grouped_canary_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                            uint64_t n_canaries_total, uint32_t S, int64_t *__restrict__ u2_out,
+                            int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
+                            int32_t *status) {
+  constexpr int kPerWarp = 32 / G;
+  const int lane = threadIdx.x & 31;
+  const uint64_t step = (uint64_t)gridDim.x * kRankWarps * kPerWarp;
+  bool saw_nan = false;
+  for (uint64_t o0 = ((uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5)) * kPerWarp;
+       o0 < n_canaries_total; o0 += step) {
+    const uint64_t o = o0 + (uint64_t)(lane / G);
+    const bool active = o < n_canaries_total;
+    long long g, e;
+    int nm, nb;
+    group_counts<G>(scores, labels, o, active, S, lane, g, e, nm, nb, saw_nan);
+    if ((lane & (G - 1)) == 0 && active) {
+      u2_out[o] = 2 * g + e;
+      if (gt_out) gt_out[o] = g;
+      if (eq_out) eq_out[o] = e;
+    }
+  }
+  if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
+    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+}
+
 // Small batches (few configurations): the same per-canary counts with one
 // warp per (configuration, canary) across the whole grid, then one block
 // per configuration combines them.  Integer sums make both paths give the
@@ -484,21 +631,53 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
                          int32_t *status, cudaStream_t stream) {
   DeviceInfo info;
   if (!device_info(&info)) return cudaGetLastError();
-  if ((uint64_t)C >= 2ull * (uint64_t)info.sm_count) {
-    // many configurations: one block each, canaries and combine fused
-    uint64_t grid = (uint64_t)info.sm_count * 8;
-    if (grid > C) grid = C;
-    auroc_kernel<<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, u2, gt, eq,
-                                                              auroc, status);
-    return cudaGetLastError();
-  }
-  // few configurations: spread the canaries over the GPU, then combine
+  const bool many = (uint64_t)C >= 2ull * (uint64_t)info.sm_count;
   const uint64_t total = (uint64_t)C * N;
-  uint64_t blocks = (total + kRankWarps - 1) / kRankWarps;
   const uint64_t cap = (uint64_t)info.sm_count * 8;
-  if (blocks > cap) blocks = cap;
-  auroc_canary_kernel<<<(unsigned)blocks, kRankThreads, 0, stream>>>(scores, labels, total, S, u2,
-                                                                     gt, eq, status);
+  if (S > 32) {
+    // wide pipelines: one warp per canary, stages strided over the lanes
+    if (many) {
+      const uint64_t grid = cap < C ? cap : C;
+      auroc_kernel<<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, u2, gt,
+                                                                eq, auroc, status);
+      return cudaGetLastError();
+    }
+    uint64_t blocks = (total + kRankWarps - 1) / kRankWarps;
+    if (blocks > cap) blocks = cap;
+    auroc_canary_kernel<<<(unsigned)blocks, kRankThreads, 0, stream>>>(scores, labels, total, S, u2,
+                                                                       gt, eq, status);
+  } else {
+    const int G = S <= 2 ? 2 : S <= 4 ? 4 : S <= 8 ? 8 : S <= 16 ? 16 : 32;
+    const uint64_t per_block = (uint64_t)kRankWarps * (32 / G);
+    if (many) {
+      const uint64_t grid = cap < C ? cap : C;
+#define CG_GROUPED(GG)                                                                         \
+  auroc_grouped_kernel<GG><<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, \
+                                                                       u2, gt, eq, auroc, status)
+      switch (G) {
+        case 2: CG_GROUPED(2); break;
+        case 4: CG_GROUPED(4); break;
+        case 8: CG_GROUPED(8); break;
+        case 16: CG_GROUPED(16); break;
+        default: CG_GROUPED(32); break;
+      }
+#undef CG_GROUPED
+      return cudaGetLastError();
+    }
+    uint64_t blocks = (total + per_block - 1) / per_block;
+    if (blocks > cap) blocks = cap;
+#define CG_GROUPED_CANARY(GG)                                                              \
+  auroc_grouped_canary_kernel<GG><<<(unsigned)blocks, kRankThreads, 0, stream>>>(           \
+      scores, labels, total, S, u2, gt, eq, status)
+    switch (G) {
+      case 2: CG_GROUPED_CANARY(2); break;
+      case 4: CG_GROUPED_CANARY(4); break;
+      case 8: CG_GROUPED_CANARY(8); break;
+      case 16: CG_GROUPED_CANARY(16); break;
+      default: CG_GROUPED_CANARY(32); break;
+    }
+#undef CG_GROUPED_CANARY
+  }
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
   auroc_config_kernel<<<C, kRankThreads, 0, stream>>>(labels, C, N, S, u2, auroc);
