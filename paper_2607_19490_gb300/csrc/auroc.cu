@@ -157,38 +157,60 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
 // canary, so one warp ranks 32 / G canaries at once; the shuffles run
 // within each G-lane group (width G).  Lane j of a group holds stage j.
 template <int G>
-__device__ __forceinline__ void group_counts(const float *__restrict__ scores,
-                                             const int8_t *__restrict__ labels, uint64_t o,
-                                             bool active, uint32_t S, int lane, long long &g,
-                                             long long &e, int &nm, int &nb, bool &saw_nan) {
+__device__ __forceinline__ void group_load(const float *__restrict__ scores,
+                                           const int8_t *__restrict__ labels, uint64_t o,
+                                           bool active, uint32_t S, int lane, float &m, int &l) {
   const int sub = lane & (G - 1);
   const bool in = active && (uint32_t)sub < S;
-  const float m = in ? scores[o * S + sub] : 0.f;
-  const int l = in ? (int)labels[o * S + sub] : -1;
+  m = in ? scores[o * S + sub] : 0.f;
+  l = in ? (int)labels[o * S + sub] : -1;
+}
+
+template <int G>
+__device__ __forceinline__ void group_rank(float m, int l, int lane, long long &g, long long &e,
+                                           int &nm, int &nb, bool &saw_nan) {
   if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
-  int lg = 0, le = 0;
-  for (uint32_t k = 0; k < S; ++k) {
-    const float mk = __shfl_sync(0xFFFFFFFFu, m, (int)k, G);
-    const int lk = __shfl_sync(0xFFFFFFFFu, l, (int)k, G);
-    if (l == 1 && lk == 0) {
-      lg += (m > mk);
-      le += (m == mk);
-    }
-  }
   const unsigned shift = (unsigned)(lane & ~(G - 1));
   const unsigned gmask = (G == 32) ? 0xFFFFFFFFu : ((1u << G) - 1u);
-  nm = __popc((__ballot_sync(0xFFFFFFFFu, l == 1) >> shift) & gmask);
-  nb = __popc((__ballot_sync(0xFFFFFFFFu, l == 0) >> shift) & gmask);
-#pragma unroll
-  for (int off = G / 2; off > 0; off >>= 1) {
-    lg += __shfl_xor_sync(0xFFFFFFFFu, lg, off, G);
-    le += __shfl_xor_sync(0xFFFFFFFFu, le, off, G);
+  const unsigned mal = (__ballot_sync(0xFFFFFFFFu, l == 1) >> shift) & gmask;
+  const unsigned ben = (__ballot_sync(0xFFFFFFFFu, l == 0) >> shift) & gmask;
+  nm = __popc(mal);
+  nb = __popc(ben);
+  // Each malicious stage of the group broadcasts its score once; every
+  // benign lane compares, and the group's counts are population counts of
+  // the warp's votes.  The loop runs to the largest malicious count of any
+  // group in the warp so that every lane votes in every round.
+  const int rounds = __reduce_max_sync(0xFFFFFFFFu, (unsigned)nm);
+  unsigned rest = mal;
+  int lg = 0, le = 0;
+  for (int r = 0; r < rounds; ++r) {
+    const bool have = rest != 0u;
+    const int k = have ? (int)shift + __ffs(rest) - 1 : lane;
+    rest &= rest - 1u;
+    const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
+    const unsigned gtb = __ballot_sync(0xFFFFFFFFu, have && l == 0 && mk > m);
+    const unsigned eqb = __ballot_sync(0xFFFFFFFFu, have && l == 0 && mk == m);
+    lg += __popc((gtb >> shift) & gmask);
+    le += __popc((eqb >> shift) & gmask);
   }
   g = lg;
   e = le;
 }
 
-// One block per configuration (many configurations).
+template <int G>
+__device__ __forceinline__ void group_counts(const float *__restrict__ scores,
+                                             const int8_t *__restrict__ labels, uint64_t o,
+                                             bool active, uint32_t S, int lane, long long &g,
+                                             long long &e, int &nm, int &nb, bool &saw_nan) {
+  float m;
+  int l;
+  group_load<G>(scores, labels, o, active, S, lane, m, l);
+  group_rank<G>(m, l, lane, g, e, nm, nb, saw_nan);
+}
+
+// One block per configuration (many configurations).  Each warp first loads
+// kPrefetch groups of canaries, then ranks them (more loads in flight).
+constexpr int kPrefetch = 4;
 template <int G>
 __global__ void __launch_bounds__(kRankThreads)
 auroc_grouped_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
@@ -202,24 +224,35 @@ auroc_grouped_kernel(const float *__restrict__ scores, const int8_t *__restrict_
   for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
     long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
     bool saw_nan = false;
-    for (uint32_t n0 = (uint32_t)warp * kPerWarp; n0 < N; n0 += kRankWarps * kPerWarp) {
-      const uint32_t n = n0 + (uint32_t)(lane / G);
-      const bool active = n < N;
-      const uint64_t o = (uint64_t)c * N + n;
-      long long g, e;
-      int nm, nb;
-      group_counts<G>(scores, labels, o, active, S, lane, g, e, nm, nb, saw_nan);
-      if (leader && active) {
-        const long long u2 = 2 * g + e;
-        u2_out[o] = u2;
-        if (gt_out) gt_out[o] = g;
-        if (eq_out) eq_out[o] = e;
-        const long long pairs = (long long)nm * nb;
-        if (pairs > 0) {
-          total += u2;
-          valid += 1;
-          pmin = min(pmin, pairs);
-          pmax = max(pmax, pairs);
+    for (uint32_t n0 = (uint32_t)warp * kPerWarp; n0 < N;
+         n0 += kRankWarps * kPerWarp * kPrefetch) {
+      float mv[kPrefetch];
+      int lv[kPrefetch];
+#pragma unroll
+      for (int u = 0; u < kPrefetch; ++u) {
+        const uint32_t n = n0 + (uint32_t)(u * kRankWarps * kPerWarp) + (uint32_t)(lane / G);
+        group_load<G>(scores, labels, (uint64_t)c * N + n, n < N, S, lane, mv[u], lv[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kPrefetch; ++u) {
+        const uint32_t n = n0 + (uint32_t)(u * kRankWarps * kPerWarp) + (uint32_t)(lane / G);
+        const bool active = n < N;
+        const uint64_t o = (uint64_t)c * N + n;
+        long long g, e;
+        int nm, nb;
+        group_rank<G>(mv[u], lv[u], lane, g, e, nm, nb, saw_nan);
+        if (leader && active) {
+          const long long u2 = 2 * g + e;
+          u2_out[o] = u2;
+          if (gt_out) gt_out[o] = g;
+          if (eq_out) eq_out[o] = e;
+          const long long pairs = (long long)nm * nb;
+          if (pairs > 0) {
+            total += u2;
+            valid += 1;
+            pmin = min(pmin, pairs);
+            pmax = max(pmax, pairs);
+          }
         }
       }
     }
@@ -270,6 +303,91 @@ auroc_grouped_kernel(const float *__restrict__ scores, const int8_t *__restrict_
     }
     __syncthreads();
   }
+}
+
+// One warp per configuration (large batches): the warp ranks the
+// configuration's canaries 32 / G at a time with kPrefetch groups of loads
+// in flight, reduces the integer sums with shuffles, and lane 0 forms A-hat.
+// No block-wide barrier anywhere, so the warps of a block never wait for
+// one another.
+template <int G>
+__global__ void __launch_bounds__(kRankThreads)
+auroc_warp_config_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                         uint32_t C, uint32_t N, uint32_t S, int64_t *__restrict__ u2_out,
+                         int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
+                         double *__restrict__ auroc, int32_t *status) {
+  constexpr int kPerWarp = 32 / G;
+  const int lane = threadIdx.x & 31;
+  const bool leader = (lane & (G - 1)) == 0;
+  const uint64_t warps = (uint64_t)gridDim.x * kRankWarps;
+  bool saw_nan = false;
+  for (uint64_t c = (uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5); c < C; c += warps) {
+    long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
+    for (uint32_t n0 = 0; n0 < N; n0 += kPerWarp * kPrefetch) {
+      float mv[kPrefetch];
+      int lv[kPrefetch];
+#pragma unroll
+      for (int u = 0; u < kPrefetch; ++u) {
+        const uint32_t n = n0 + (uint32_t)(u * kPerWarp) + (uint32_t)(lane / G);
+        group_load<G>(scores, labels, c * N + n, n < N, S, lane, mv[u], lv[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kPrefetch; ++u) {
+        const uint32_t n = n0 + (uint32_t)(u * kPerWarp) + (uint32_t)(lane / G);
+        long long g, e;
+        int nm, nb;
+        group_rank<G>(mv[u], lv[u], lane, g, e, nm, nb, saw_nan);
+        if (leader && n < N) {
+          const uint64_t o = c * N + n;
+          const long long u2 = 2 * g + e;
+          u2_out[o] = u2;
+          if (gt_out) gt_out[o] = g;
+          if (eq_out) eq_out[o] = e;
+          const long long pairs = (long long)nm * nb;
+          if (pairs > 0) {
+            total += u2;
+            valid += 1;
+            pmin = min(pmin, pairs);
+            pmax = max(pmax, pairs);
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      total += __shfl_xor_sync(0xFFFFFFFFu, total, off);
+      valid += __shfl_xor_sync(0xFFFFFFFFu, valid, off);
+      pmin = min(pmin, __shfl_xor_sync(0xFFFFFFFFu, pmin, off));
+      pmax = max(pmax, __shfl_xor_sync(0xFFFFFFFFu, pmax, off));
+    }
+    __syncwarp();   // the leaders' u2 writes are visible to lane 0 below
+    if (lane == 0) {
+      double A;
+      if (valid == 0) {
+        A = NAN;
+      } else if (pmin == pmax) {
+        A = __ddiv_rn((double)total, (double)(2 * pmin * valid));
+      } else {
+        // pair counts differ between canaries: per-canary ratios in order
+        double acc = 0.0;
+        for (uint32_t n = 0; n < N; ++n) {
+          const int8_t *l = labels + (c * N + n) * S;
+          long long nm = 0, nb = 0;
+          for (uint32_t s = 0; s < S; ++s) {
+            nm += (l[s] == 1);
+            nb += (l[s] == 0);
+          }
+          if (nm * nb == 0) continue;
+          acc = __dadd_rn(acc, __ddiv_rn((double)u2_out[c * N + n], (double)(2 * nm * nb)));
+        }
+        A = __ddiv_rn(acc, (double)valid);
+      }
+      auroc[c] = A;
+    }
+    __syncwarp();
+  }
+  if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
+    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
 // Canary-parallel counts for few configurations (combine: auroc_config_kernel).
@@ -650,10 +768,11 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
     const int G = S <= 2 ? 2 : S <= 4 ? 4 : S <= 8 ? 8 : S <= 16 ? 16 : 32;
     const uint64_t per_block = (uint64_t)kRankWarps * (32 / G);
     if (many) {
-      const uint64_t grid = cap < C ? cap : C;
-#define CG_GROUPED(GG)                                                                         \
-  auroc_grouped_kernel<GG><<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, S, \
-                                                                       u2, gt, eq, auroc, status)
+      const uint64_t grid = ((uint64_t)C + kRankWarps - 1) / kRankWarps;   // a warp each
+#define CG_GROUPED(GG)                                                                          \
+  auroc_warp_config_kernel<GG><<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, \
+                                                                           S, u2, gt, eq, auroc, \
+                                                                           status)
       switch (G) {
         case 2: CG_GROUPED(2); break;
         case 4: CG_GROUPED(4); break;
