@@ -349,7 +349,9 @@ def run_ours(args, ranks: Ranks):
     outs = {k: torch.empty((1, N), dtype=torch.int64, device=dev) for k in ("u2", "gt", "eq")}
     outs_c = {k: torch.empty((1, N), dtype=torch.int64, device=dev) for k in ("u2", "gt", "eq")}
     auroc = torch.empty((2,), dtype=torch.float64, device=dev)
-    launches_per_step = 5          # drift partial + finalize, control labels, 2 x AUROC
+    # drift (pipeline kernel + finalize), control labels, and two AUROC calls
+    # of one configuration (canary-parallel counts + per-configuration combine)
+    launches_per_step = 2 + 1 + 2 * 2
 
     algo = {"auto": None, "stream": cg.DRIFT_STREAM, "bulk": cg.DRIFT_BULK,
             "bulk2": cg.DRIFT_BULK_2CTA}[args.drift_algo]
