@@ -331,6 +331,16 @@ cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels,
                           double *d_auroc, int32_t *d_status, cg_stream_t stream);
 
 /*
+ * Diagnostic of the failure path of the library's device waits (the
+ * bulk-copy drift pipeline waits on mbarriers with a time limit): one warp
+ * waits on an mbarrier phase that nothing completes, gives up after
+ * limit_us microseconds (1 .. 10^7) and raises CG_DEVFLAG_TIMEOUT in
+ * d_status (required), which cg_read_status then reports as
+ * CG_ERR_TIMEOUT.  The device stays usable afterwards.
+ */
+cg_status cg_selftest_bounded_wait(uint32_t limit_us, int32_t *d_status, cg_stream_t stream);
+
+/*
  * Synchronise `stream`, read the device status word and map it: 0 ->
  * CG_OK, else the first of CG_ERR_TIMEOUT, CG_ERR_NAN_SCORE,
  * CG_ERR_NO_BENIGN that is set.  The raw word goes to *h_word if non-NULL.

@@ -22,7 +22,7 @@ __all__ = [
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
     "cg_drift_scores_ex", "cg_drift_scores_host", "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
-    "cg_random_scores", "cg_auroc_pooled", "cg_generate_propagating",
+    "cg_random_scores", "cg_auroc_pooled", "cg_generate_propagating", "cg_selftest_bounded_wait",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
     "TAMPER_SIGNFLIP_FULL", "TAMPER_SCALE",
 ]
@@ -106,6 +106,7 @@ def load() -> ctypes.CDLL:
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
             "cg_auroc": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
             "cg_auroc_pooled": ([P, P, u32, u32, u32, P, P, P, P, P, P], ctypes.c_int),
+            "cg_selftest_bounded_wait": ([u32, P, P], ctypes.c_int),
             "cg_read_status": ([P, P, ctypes.POINTER(i32)], ctypes.c_int),
         }
         for name, (args, res) in sigs.items():
@@ -453,6 +454,14 @@ def cg_auroc_pooled(scores, labels, u2=None, n_mal=None, n_ben=None, auroc=None,
                                   _ptr(n_ben), _ptr(auroc), _ptr(status), _stream(stream)),
            "cg_auroc_pooled")
     return {"u2": u2, "n_mal": n_mal, "n_ben": n_ben, "auroc": auroc}
+
+
+def cg_selftest_bounded_wait(limit_us, status, stream=None):
+    """Run the bounded-wait diagnostic; returns nothing (read `status` afterwards)."""
+    torch = _torch()
+    _cuda(status, "status", (torch.int32,))
+    _check(load().cg_selftest_bounded_wait(int(limit_us), _ptr(status), _stream(stream)),
+           "cg_selftest_bounded_wait")
 
 
 def cg_read_status(status, stream=None):

@@ -2,10 +2,11 @@
 // (Eq. 5, ties counted as one half) and their mean over canaries (Eq. 6),
 // plus the labels of the scrambled-label negative control (Sec. 4.5).
 //
-// auroc_kernel: one block per configuration, one warp per canary at a time.
-// For S <= 32 each lane holds one stage's score and label and the warp
-// compares every (malicious, benign) pair through shuffles; larger S is
-// strided over the lanes with the benign side read from global memory.
+// auroc_warp_config_kernel (many configurations) and
+// auroc_grouped_canary_kernel + auroc_config_kernel (few): S <= 32, one
+// G-lane group per canary, the malicious stages broadcast and the benign
+// stages vote.  auroc_kernel / auroc_canary_kernel: S > 32, one warp per
+// canary with the stages strided over the lanes.
 // Counts are integers (exact in any order); the configuration's A-hat is
 // one fp64 division of exact integers when every canary has the same pair
 // count, else the per-canary ratios added in canary order by one thread.
@@ -21,6 +22,60 @@ constexpr int kRankThreads = 256;
 constexpr int kRankWarps = kRankThreads / 32;
 
 __device__ __forceinline__ bool is_nan_f(float x) { return x != x; }
+
+__device__ __forceinline__ void canary_counts(const float *m_all, const int8_t *l_all, uint32_t S,
+                                              int lane, long long &g, long long &e, int &nm,
+                                              int &nb, bool &saw_nan) {
+  g = 0;
+  e = 0;
+  if (S <= 32) {
+    const bool in = (uint32_t)lane < S;
+    const float m = in ? m_all[lane] : 0.f;
+    const int l = in ? (int)l_all[lane] : -1;
+    if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
+    int lg = 0, le = 0;
+    for (uint32_t k = 0; k < S; ++k) {
+      const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
+      const int lk = __shfl_sync(0xFFFFFFFFu, l, k);
+      if (l == 1 && lk == 0) {
+        lg += (m > mk);
+        le += (m == mk);
+      }
+    }
+    nm = __popc(__ballot_sync(0xFFFFFFFFu, l == 1));
+    nb = __popc(__ballot_sync(0xFFFFFFFFu, l == 0));
+    g = lg;
+    e = le;
+  } else {
+    int lm = 0, lb = 0;
+    for (uint32_t i = lane; i < S; i += 32) {
+      const float m = m_all[i];
+      const int l = (int)l_all[i];
+      if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
+      lm += (l == 1);
+      lb += (l == 0);
+      if (l != 1) continue;
+      for (uint32_t j = 0; j < S; ++j) {
+        if (l_all[j] != 0) continue;
+        const float mj = m_all[j];
+        g += (m > mj);
+        e += (m == mj);
+      }
+    }
+    nm = lm;
+    nb = lb;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      nm += __shfl_xor_sync(0xFFFFFFFFu, nm, off);
+      nb += __shfl_xor_sync(0xFFFFFFFFu, nb, off);
+    }
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    g += __shfl_xor_sync(0xFFFFFFFFu, g, off);
+    e += __shfl_xor_sync(0xFFFFFFFFu, e, off);
+  }
+}
 
 __global__ void __launch_bounds__(kRankThreads)
 auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels, uint32_t C,
@@ -38,59 +93,9 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
     bool saw_nan = false;
     for (uint32_t n = warp; n < N; n += kRankWarps) {
       const uint64_t base = ((uint64_t)c * N + n) * S;
-      long long g = 0, e = 0;
-      int nm = 0, nb = 0;
-      if (S <= 32) {
-        const bool in = (uint32_t)lane < S;
-        const float m = in ? scores[base + lane] : 0.f;
-        const int l = in ? (int)labels[base + lane] : -1;
-        const bool labelled = (l == 0 || l == 1);
-        if (labelled && is_nan_f(m)) saw_nan = true;
-        int lg = 0, le = 0;
-        for (uint32_t k = 0; k < S; ++k) {
-          const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
-          const int lk = __shfl_sync(0xFFFFFFFFu, l, k);
-          if (l == 1 && lk == 0) {
-            lg += (m > mk);
-            le += (m == mk);
-          }
-        }
-        nm = __popc(__ballot_sync(0xFFFFFFFFu, l == 1));
-        nb = __popc(__ballot_sync(0xFFFFFFFFu, l == 0));
-        g = lg;
-        e = le;
-      } else {
-        long long lg = 0, le = 0;
-        int lm = 0, lb = 0;
-        for (uint32_t i = lane; i < S; i += 32) {
-          const float m = scores[base + i];
-          const int l = (int)labels[base + i];
-          if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
-          lm += (l == 1);
-          lb += (l == 0);
-          if (l != 1) continue;
-          for (uint32_t j = 0; j < S; ++j) {
-            if (labels[base + j] != 0) continue;
-            const float mj = scores[base + j];
-            lg += (m > mj);
-            le += (m == mj);
-          }
-        }
-        g = lg;
-        e = le;
-        nm = lm;
-        nb = lb;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) {
-          nm += __shfl_xor_sync(0xFFFFFFFFu, nm, off);
-          nb += __shfl_xor_sync(0xFFFFFFFFu, nb, off);
-        }
-      }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        g += __shfl_xor_sync(0xFFFFFFFFu, g, off);
-        e += __shfl_xor_sync(0xFFFFFFFFu, e, off);
-      }
+      long long g, e;
+      int nm, nb;
+      canary_counts(scores + base, labels + base, S, lane, g, e, nm, nb, saw_nan);
       if (lane == 0) {
         const uint64_t o = (uint64_t)c * N + n;
         const long long u2 = 2 * g + e;
@@ -208,102 +213,8 @@ __device__ __forceinline__ void group_counts(const float *__restrict__ scores,
   group_rank<G>(m, l, lane, g, e, nm, nb, saw_nan);
 }
 
-// One block per configuration (many configurations).  Each warp first loads
-// kPrefetch groups of canaries, then ranks them (more loads in flight).
+// Loads of this many canary groups are issued before any is ranked.
 constexpr int kPrefetch = 4;
-template <int G>
-__global__ void __launch_bounds__(kRankThreads)
-auroc_grouped_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
-                     uint32_t C, uint32_t N, uint32_t S, int64_t *__restrict__ u2_out,
-                     int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
-                     double *__restrict__ auroc, int32_t *status) {
-  constexpr int kPerWarp = 32 / G;
-  __shared__ long long red[kRankWarps][4];
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const bool leader = (lane & (G - 1)) == 0;
-  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
-    long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
-    bool saw_nan = false;
-    for (uint32_t n0 = (uint32_t)warp * kPerWarp; n0 < N;
-         n0 += kRankWarps * kPerWarp * kPrefetch) {
-      float mv[kPrefetch];
-      int lv[kPrefetch];
-#pragma unroll
-      for (int u = 0; u < kPrefetch; ++u) {
-        const uint32_t n = n0 + (uint32_t)(u * kRankWarps * kPerWarp) + (uint32_t)(lane / G);
-        group_load<G>(scores, labels, (uint64_t)c * N + n, n < N, S, lane, mv[u], lv[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < kPrefetch; ++u) {
-        const uint32_t n = n0 + (uint32_t)(u * kRankWarps * kPerWarp) + (uint32_t)(lane / G);
-        const bool active = n < N;
-        const uint64_t o = (uint64_t)c * N + n;
-        long long g, e;
-        int nm, nb;
-        group_rank<G>(mv[u], lv[u], lane, g, e, nm, nb, saw_nan);
-        if (leader && active) {
-          const long long u2 = 2 * g + e;
-          u2_out[o] = u2;
-          if (gt_out) gt_out[o] = g;
-          if (eq_out) eq_out[o] = e;
-          const long long pairs = (long long)nm * nb;
-          if (pairs > 0) {
-            total += u2;
-            valid += 1;
-            pmin = min(pmin, pairs);
-            pmax = max(pmax, pairs);
-          }
-        }
-      }
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      total += __shfl_down_sync(0xFFFFFFFFu, total, off);
-      valid += __shfl_down_sync(0xFFFFFFFFu, valid, off);
-      pmin = min(pmin, __shfl_down_sync(0xFFFFFFFFu, pmin, off));
-      pmax = max(pmax, __shfl_down_sync(0xFFFFFFFFu, pmax, off));
-    }
-    if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
-      atomicOr(status, CG_DEVFLAG_NAN_SCORE);
-    if (lane == 0) {
-      red[warp][0] = total;
-      red[warp][1] = valid;
-      red[warp][2] = pmin;
-      red[warp][3] = pmax;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      for (int w = 1; w < kRankWarps; ++w) {
-        red[0][0] += red[w][0];
-        red[0][1] += red[w][1];
-        red[0][2] = min(red[0][2], red[w][2]);
-        red[0][3] = max(red[0][3], red[w][3]);
-      }
-      const long long T = red[0][0], V = red[0][1];
-      double A;
-      if (V == 0) {
-        A = NAN;
-      } else if (red[0][2] == red[0][3]) {
-        A = __ddiv_rn((double)T, (double)(2 * red[0][2] * V));
-      } else {
-        double acc = 0.0;
-        for (uint32_t n = 0; n < N; ++n) {
-          const int8_t *l = labels + ((uint64_t)c * N + n) * S;
-          long long nm = 0, nb = 0;
-          for (uint32_t s = 0; s < S; ++s) {
-            nm += (l[s] == 1);
-            nb += (l[s] == 0);
-          }
-          if (nm * nb == 0) continue;
-          acc = __dadd_rn(acc, __ddiv_rn((double)u2_out[(uint64_t)c * N + n], (double)(2 * nm * nb)));
-        }
-        A = __ddiv_rn(acc, (double)V);
-      }
-      auroc[c] = A;
-    }
-    __syncthreads();
-  }
-}
 
 // One warp per configuration (large batches): the warp ranks the
 // configuration's canaries 32 / G at a time with kPrefetch groups of loads
@@ -422,60 +333,6 @@ auroc_grouped_canary_kernel(const float *__restrict__ scores, const int8_t *__re
 // warp per (configuration, canary) across the whole grid, then one block
 // per configuration combines them.  Integer sums make both paths give the
 // same bits.
-__device__ __forceinline__ void canary_counts(const float *m_all, const int8_t *l_all, uint32_t S,
-                                              int lane, long long &g, long long &e, int &nm,
-                                              int &nb, bool &saw_nan) {
-  g = 0;
-  e = 0;
-  if (S <= 32) {
-    const bool in = (uint32_t)lane < S;
-    const float m = in ? m_all[lane] : 0.f;
-    const int l = in ? (int)l_all[lane] : -1;
-    if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
-    int lg = 0, le = 0;
-    for (uint32_t k = 0; k < S; ++k) {
-      const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
-      const int lk = __shfl_sync(0xFFFFFFFFu, l, k);
-      if (l == 1 && lk == 0) {
-        lg += (m > mk);
-        le += (m == mk);
-      }
-    }
-    nm = __popc(__ballot_sync(0xFFFFFFFFu, l == 1));
-    nb = __popc(__ballot_sync(0xFFFFFFFFu, l == 0));
-    g = lg;
-    e = le;
-  } else {
-    int lm = 0, lb = 0;
-    for (uint32_t i = lane; i < S; i += 32) {
-      const float m = m_all[i];
-      const int l = (int)l_all[i];
-      if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
-      lm += (l == 1);
-      lb += (l == 0);
-      if (l != 1) continue;
-      for (uint32_t j = 0; j < S; ++j) {
-        if (l_all[j] != 0) continue;
-        const float mj = m_all[j];
-        g += (m > mj);
-        e += (m == mj);
-      }
-    }
-    nm = lm;
-    nb = lb;
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      nm += __shfl_xor_sync(0xFFFFFFFFu, nm, off);
-      nb += __shfl_xor_sync(0xFFFFFFFFu, nb, off);
-    }
-  }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    g += __shfl_xor_sync(0xFFFFFFFFu, g, off);
-    e += __shfl_xor_sync(0xFFFFFFFFu, e, off);
-  }
-}
-
 __global__ void __launch_bounds__(kRankThreads)
 auroc_canary_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
                     uint64_t n_canaries_total, uint32_t S, int64_t *__restrict__ u2_out,

@@ -357,6 +357,12 @@ cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels, uint32_
                                            (cudaStream_t)stream));
 }
 
+cg_status cg_selftest_bounded_wait(uint32_t limit_us, int32_t *d_status, cg_stream_t stream) {
+  if (!d_status || limit_us == 0 || limit_us > 10u * 1000u * 1000u) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_status, 4)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_bounded_wait_probe(limit_us, d_status, (cudaStream_t)stream));
+}
+
 cg_status cg_read_status(const int32_t *d_status, cg_stream_t stream, int32_t *h_word) {
   if (!d_status) return CG_ERR_INVALID_ARG;
   int32_t w = 0;

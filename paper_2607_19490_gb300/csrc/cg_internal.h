@@ -39,6 +39,7 @@ cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, ui
                          uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
                          cudaStream_t stream);
 
+cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream);
 bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len);
 cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
                               uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,

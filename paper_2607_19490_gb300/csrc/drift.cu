@@ -269,8 +269,9 @@ __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
 }
 
 // true once the phase with the given parity has completed; false after
-// kBulkWaitNs without completion
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+// limit_ns of global-timer time without completion
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity,
+                                          unsigned long long limit_ns = kBulkWaitNs) {
   const unsigned long long t0 = global_ns();
   for (uint32_t it = 0;; ++it) {
     uint32_t done;
@@ -282,7 +283,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
         : "r"(bar), "r"(parity)
         : "memory");
     if (done) return true;
-    if ((it & 63u) == 63u && global_ns() - t0 > kBulkWaitNs) return false;
+    if ((it & 63u) == 63u && global_ns() - t0 > limit_ns) return false;
   }
 }
 
@@ -443,6 +444,22 @@ drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ r
 
 }  // namespace
 
+// Diagnostic for the bounded wait: one warp waits on a phase of an mbarrier
+// that nothing arrives at.  The wait must give up after limit_ns and raise
+// CG_DEVFLAG_TIMEOUT; no copy is in flight, so the block can leave.
+__global__ void bounded_wait_probe_kernel(unsigned long long limit_ns, int32_t *status) {
+  __shared__ __align__(8) unsigned long long bar;
+  const uint32_t b = (uint32_t)__cvta_generic_to_shared(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(b, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const bool done = mbar_wait(b, 0u, limit_ns);
+  if (!__all_sync(0xFFFFFFFFu, done) && threadIdx.x == 0 && status)
+    atomicOr(status, CG_DEVFLAG_TIMEOUT);
+}
+
 template <int NS>
 static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t seg_len,
                                uint64_t cps, uint64_t n_items, float4 *partials, int32_t *status,
@@ -491,6 +508,11 @@ cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t 
   }
   if (err != cudaSuccess) return err;
   return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
+}
+
+cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream) {
+  bounded_wait_probe_kernel<<<1, 32, 0, stream>>>(1000ull * limit_us, status);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
