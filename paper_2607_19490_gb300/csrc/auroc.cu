@@ -2,11 +2,11 @@
 // (Eq. 5, ties counted as one half) and their mean over canaries (Eq. 6),
 // plus the labels of the scrambled-label negative control (Sec. 4.5).
 //
-// auroc_warp_config_kernel (many configurations) and
-// auroc_grouped_canary_kernel + auroc_config_kernel (few): S <= 32, one
-// G-lane group per canary, the malicious stages broadcast and the benign
-// stages vote.  auroc_kernel / auroc_canary_kernel: S > 32, one warp per
-// canary with the stages strided over the lanes.
+// S <= 32: one lane per canary -- auroc_lane_config_kernel (many
+// configurations: a warp per configuration) or auroc_lane_canary_kernel +
+// auroc_config_kernel (few: lanes over all canaries, then a combine).
+// S > 32: one warp per canary with the stages strided over the lanes
+// (auroc_kernel / auroc_canary_kernel).
 // Counts are integers (exact in any order); the configuration's A-hat is
 // one fp64 division of exact integers when every canary has the same pair
 // count, else the per-canary ratios added in canary order by one thread.
@@ -22,6 +22,28 @@ constexpr int kRankThreads = 256;
 constexpr int kRankWarps = kRankThreads / 32;
 
 __device__ __forceinline__ bool is_nan_f(float x) { return x != x; }
+
+// A-hat of configuration c from its integer sums (Eq. 6): one fp64 division
+// when every canary with a pair has the same pair count (pmin == pmax),
+// else the per-canary ratios added in canary order; NaN without a pair.
+__device__ double combine_auroc(const int8_t *__restrict__ labels, uint64_t c, uint32_t N,
+                                uint32_t S, const int64_t *__restrict__ u2, long long total,
+                                long long valid, long long pmin, long long pmax) {
+  if (valid == 0) return NAN;
+  if (pmin == pmax) return __ddiv_rn((double)total, (double)(2 * pmin * valid));
+  double acc = 0.0;
+  for (uint32_t n = 0; n < N; ++n) {
+    const int8_t *l = labels + (c * N + n) * S;
+    long long nm = 0, nb = 0;
+    for (uint32_t s = 0; s < S; ++s) {
+      nm += (l[s] == 1);
+      nb += (l[s] == 0);
+    }
+    if (nm * nb == 0) continue;
+    acc = __dadd_rn(acc, __ddiv_rn((double)u2[c * N + n], (double)(2 * nm * nb)));
+  }
+  return __ddiv_rn(acc, (double)valid);
+}
 
 __device__ __forceinline__ void canary_counts(const float *m_all, const int8_t *l_all, uint32_t S,
                                               int lane, long long &g, long long &e, int &nm,
@@ -158,110 +180,88 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
   }
 }
 
-// Grouped ranking for S <= 32: G = the next power of two >= S lanes per
-// canary, so one warp ranks 32 / G canaries at once; the shuffles run
-// within each G-lane group (width G).  Lane j of a group holds stage j.
-template <int G>
-__device__ __forceinline__ void group_load(const float *__restrict__ scores,
-                                           const int8_t *__restrict__ labels, uint64_t o,
-                                           bool active, uint32_t S, int lane, float &m, int &l) {
-  const int sub = lane & (G - 1);
-  const bool in = active && (uint32_t)sub < S;
-  m = in ? scores[o * S + sub] : 0.f;
-  l = in ? (int)labels[o * S + sub] : -1;
-}
-
-template <int G>
-__device__ __forceinline__ void group_rank(float m, int l, int lane, long long &g, long long &e,
-                                           int &nm, int &nb, bool &saw_nan) {
-  if ((l == 0 || l == 1) && is_nan_f(m)) saw_nan = true;
-  const unsigned shift = (unsigned)(lane & ~(G - 1));
-  const unsigned gmask = (G == 32) ? 0xFFFFFFFFu : ((1u << G) - 1u);
-  const unsigned mal = (__ballot_sync(0xFFFFFFFFu, l == 1) >> shift) & gmask;
-  const unsigned ben = (__ballot_sync(0xFFFFFFFFu, l == 0) >> shift) & gmask;
-  nm = __popc(mal);
-  nb = __popc(ben);
-  // Each malicious stage of the group broadcasts its score once; every
-  // benign lane compares, and the group's counts are population counts of
-  // the warp's votes.  The loop runs to the largest malicious count of any
-  // group in the warp so that every lane votes in every round.
-  const int rounds = __reduce_max_sync(0xFFFFFFFFu, (unsigned)nm);
-  unsigned rest = mal;
-  int lg = 0, le = 0;
-  for (int r = 0; r < rounds; ++r) {
-    const bool have = rest != 0u;
-    const int k = have ? (int)shift + __ffs(rest) - 1 : lane;
-    rest &= rest - 1u;
-    const float mk = __shfl_sync(0xFFFFFFFFu, m, k);
-    const unsigned gtb = __ballot_sync(0xFFFFFFFFu, have && l == 0 && mk > m);
-    const unsigned eqb = __ballot_sync(0xFFFFFFFFu, have && l == 0 && mk == m);
-    lg += __popc((gtb >> shift) & gmask);
-    le += __popc((eqb >> shift) & gmask);
+// Lane-per-canary ranking for S <= 32 (SP = S rounded up to 4, 8, 16 or
+// 32): each lane loads its canary's scores and labels into registers
+// (16-byte loads when the rows are 16-byte aligned) and counts, for every
+// malicious stage, the benign stages below it and equal to it.  A warp
+// ranks 32 canaries at once with no cross-lane traffic.
+template <int SP>
+__device__ __forceinline__ void lane_counts(const float *__restrict__ scores,
+                                            const int8_t *__restrict__ labels, uint64_t o,
+                                            uint32_t S, bool vec, long long &g, long long &e,
+                                            int &nm, int &nb, bool &saw_nan) {
+  float m[SP];
+  int l[SP];
+  const float *ms = scores + o * S;
+  const int8_t *ls = labels + o * S;
+  if (vec) {
+#pragma unroll
+    for (int k = 0; k < SP; k += 4) {
+      const float4 v = *reinterpret_cast<const float4 *>(ms + k);
+      m[k] = v.x; m[k + 1] = v.y; m[k + 2] = v.z; m[k + 3] = v.w;
+      const uint32_t w = *reinterpret_cast<const uint32_t *>(ls + k);
+      l[k] = (int)(int8_t)(w & 0xFFu);
+      l[k + 1] = (int)(int8_t)((w >> 8) & 0xFFu);
+      l[k + 2] = (int)(int8_t)((w >> 16) & 0xFFu);
+      l[k + 3] = (int)(int8_t)(w >> 24);
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < SP; ++k) {
+      m[k] = (uint32_t)k < S ? ms[k] : 0.f;
+      l[k] = (uint32_t)k < S ? (int)ls[k] : -1;
+    }
+  }
+  int lg = 0, le = 0, cm = 0, cb = 0;
+#pragma unroll
+  for (int i = 0; i < SP; ++i) {
+    if ((l[i] == 0 || l[i] == 1) && is_nan_f(m[i])) saw_nan = true;
+    cm += (l[i] == 1);
+    cb += (l[i] == 0);
+  }
+#pragma unroll
+  for (int i = 0; i < SP; ++i) {
+    if (l[i] != 1) continue;
+#pragma unroll
+    for (int j = 0; j < SP; ++j) {
+      const bool b = l[j] == 0;
+      lg += (b && m[i] > m[j]);
+      le += (b && m[i] == m[j]);
+    }
   }
   g = lg;
   e = le;
+  nm = cm;
+  nb = cb;
 }
 
-template <int G>
-__device__ __forceinline__ void group_counts(const float *__restrict__ scores,
-                                             const int8_t *__restrict__ labels, uint64_t o,
-                                             bool active, uint32_t S, int lane, long long &g,
-                                             long long &e, int &nm, int &nb, bool &saw_nan) {
-  float m;
-  int l;
-  group_load<G>(scores, labels, o, active, S, lane, m, l);
-  group_rank<G>(m, l, lane, g, e, nm, nb, saw_nan);
-}
-
-// Loads of this many canary groups are issued before any is ranked.
-constexpr int kPrefetch = 4;
-
-// One warp per configuration (large batches): the warp ranks the
-// configuration's canaries 32 / G at a time with kPrefetch groups of loads
-// in flight, reduces the integer sums with shuffles, and lane 0 forms A-hat.
-// No block-wide barrier anywhere, so the warps of a block never wait for
-// one another.
-template <int G>
+template <int SP>
 __global__ void __launch_bounds__(kRankThreads)
-auroc_warp_config_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
-                         uint32_t C, uint32_t N, uint32_t S, int64_t *__restrict__ u2_out,
-                         int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
-                         double *__restrict__ auroc, int32_t *status) {
-  constexpr int kPerWarp = 32 / G;
+auroc_lane_config_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                         uint32_t C, uint32_t N, uint32_t S, bool vec,
+                         int64_t *__restrict__ u2_out, int64_t *__restrict__ gt_out,
+                         int64_t *__restrict__ eq_out, double *__restrict__ auroc,
+                         int32_t *status) {
   const int lane = threadIdx.x & 31;
-  const bool leader = (lane & (G - 1)) == 0;
   const uint64_t warps = (uint64_t)gridDim.x * kRankWarps;
   bool saw_nan = false;
   for (uint64_t c = (uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5); c < C; c += warps) {
     long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
-    for (uint32_t n0 = 0; n0 < N; n0 += kPerWarp * kPrefetch) {
-      float mv[kPrefetch];
-      int lv[kPrefetch];
-#pragma unroll
-      for (int u = 0; u < kPrefetch; ++u) {
-        const uint32_t n = n0 + (uint32_t)(u * kPerWarp) + (uint32_t)(lane / G);
-        group_load<G>(scores, labels, c * N + n, n < N, S, lane, mv[u], lv[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < kPrefetch; ++u) {
-        const uint32_t n = n0 + (uint32_t)(u * kPerWarp) + (uint32_t)(lane / G);
-        long long g, e;
-        int nm, nb;
-        group_rank<G>(mv[u], lv[u], lane, g, e, nm, nb, saw_nan);
-        if (leader && n < N) {
-          const uint64_t o = c * N + n;
-          const long long u2 = 2 * g + e;
-          u2_out[o] = u2;
-          if (gt_out) gt_out[o] = g;
-          if (eq_out) eq_out[o] = e;
-          const long long pairs = (long long)nm * nb;
-          if (pairs > 0) {
-            total += u2;
-            valid += 1;
-            pmin = min(pmin, pairs);
-            pmax = max(pmax, pairs);
-          }
-        }
+    for (uint32_t n = lane; n < N; n += 32) {
+      const uint64_t o = c * N + n;
+      long long g, e;
+      int nm, nb;
+      lane_counts<SP>(scores, labels, o, S, vec, g, e, nm, nb, saw_nan);
+      const long long u2 = 2 * g + e;
+      u2_out[o] = u2;
+      if (gt_out) gt_out[o] = g;
+      if (eq_out) eq_out[o] = e;
+      const long long pairs = (long long)nm * nb;
+      if (pairs > 0) {
+        total += u2;
+        valid += 1;
+        pmin = min(pmin, pairs);
+        pmax = max(pmax, pairs);
       }
     }
 #pragma unroll
@@ -271,62 +271,31 @@ auroc_warp_config_kernel(const float *__restrict__ scores, const int8_t *__restr
       pmin = min(pmin, __shfl_xor_sync(0xFFFFFFFFu, pmin, off));
       pmax = max(pmax, __shfl_xor_sync(0xFFFFFFFFu, pmax, off));
     }
-    __syncwarp();   // the leaders' u2 writes are visible to lane 0 below
-    if (lane == 0) {
-      double A;
-      if (valid == 0) {
-        A = NAN;
-      } else if (pmin == pmax) {
-        A = __ddiv_rn((double)total, (double)(2 * pmin * valid));
-      } else {
-        // pair counts differ between canaries: per-canary ratios in order
-        double acc = 0.0;
-        for (uint32_t n = 0; n < N; ++n) {
-          const int8_t *l = labels + (c * N + n) * S;
-          long long nm = 0, nb = 0;
-          for (uint32_t s = 0; s < S; ++s) {
-            nm += (l[s] == 1);
-            nb += (l[s] == 0);
-          }
-          if (nm * nb == 0) continue;
-          acc = __dadd_rn(acc, __ddiv_rn((double)u2_out[c * N + n], (double)(2 * nm * nb)));
-        }
-        A = __ddiv_rn(acc, (double)valid);
-      }
-      auroc[c] = A;
-    }
+    __syncwarp();   // every lane's u2 writes are visible to lane 0 below
+    if (lane == 0) auroc[c] = combine_auroc(labels, c, N, S, u2_out, total, valid, pmin, pmax);
     __syncwarp();
   }
   if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
     atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
-// Canary-parallel counts for few configurations (combine: auroc_config_kernel).
-template <int G>
+template <int SP>
 __global__ void __launch_bounds__(kRankThreads)
-auroc_grouped_canary_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
-                            uint64_t n_canaries_total, uint32_t S, int64_t *__restrict__ u2_out,
-                            int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
-                            int32_t *status) {
-  constexpr int kPerWarp = 32 / G;
-  const int lane = threadIdx.x & 31;
-  const uint64_t step = (uint64_t)gridDim.x * kRankWarps * kPerWarp;
+auroc_lane_canary_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                         uint64_t n_canaries_total, uint32_t S, bool vec,
+                         int64_t *__restrict__ u2_out, int64_t *__restrict__ gt_out,
+                         int64_t *__restrict__ eq_out, int32_t *status) {
   bool saw_nan = false;
-  for (uint64_t o0 = ((uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5)) * kPerWarp;
-       o0 < n_canaries_total; o0 += step) {
-    const uint64_t o = o0 + (uint64_t)(lane / G);
-    const bool active = o < n_canaries_total;
+  for (uint64_t o = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; o < n_canaries_total;
+       o += (uint64_t)gridDim.x * blockDim.x) {
     long long g, e;
     int nm, nb;
-    group_counts<G>(scores, labels, o, active, S, lane, g, e, nm, nb, saw_nan);
-    if ((lane & (G - 1)) == 0 && active) {
-      u2_out[o] = 2 * g + e;
-      if (gt_out) gt_out[o] = g;
-      if (eq_out) eq_out[o] = e;
-    }
+    lane_counts<SP>(scores, labels, o, S, vec, g, e, nm, nb, saw_nan);
+    u2_out[o] = 2 * g + e;
+    if (gt_out) gt_out[o] = g;
+    if (eq_out) eq_out[o] = e;
   }
-  if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
-    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+  if (saw_nan && status) atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
 // Small batches (few configurations): the same per-canary counts with one
@@ -622,37 +591,38 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
     auroc_canary_kernel<<<(unsigned)blocks, kRankThreads, 0, stream>>>(scores, labels, total, S, u2,
                                                                        gt, eq, status);
   } else {
-    const int G = S <= 2 ? 2 : S <= 4 ? 4 : S <= 8 ? 8 : S <= 16 ? 16 : 32;
-    const uint64_t per_block = (uint64_t)kRankWarps * (32 / G);
+    const int SP = S <= 4 ? 4 : S <= 8 ? 8 : S <= 16 ? 16 : 32;
+    // 16-byte row loads only when a row is exactly SP scores and 16-byte aligned
+    const bool vec = (S == (uint32_t)SP) && ((uintptr_t)scores % 16 == 0) &&
+                     ((uintptr_t)labels % 4 == 0);
     if (many) {
       const uint64_t grid = ((uint64_t)C + kRankWarps - 1) / kRankWarps;   // a warp each
-#define CG_GROUPED(GG)                                                                          \
-  auroc_warp_config_kernel<GG><<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, \
-                                                                           S, u2, gt, eq, auroc, \
-                                                                           status)
-      switch (G) {
-        case 2: CG_GROUPED(2); break;
-        case 4: CG_GROUPED(4); break;
-        case 8: CG_GROUPED(8); break;
-        case 16: CG_GROUPED(16); break;
-        default: CG_GROUPED(32); break;
+#define CG_LANE_CONFIG(P)                                                                     \
+  auroc_lane_config_kernel<P><<<(unsigned)grid, kRankThreads, 0, stream>>>(scores, labels, C, N, \
+                                                                         S, vec, u2, gt, eq,   \
+                                                                         auroc, status)
+      switch (SP) {
+        case 4: CG_LANE_CONFIG(4); break;
+        case 8: CG_LANE_CONFIG(8); break;
+        case 16: CG_LANE_CONFIG(16); break;
+        default: CG_LANE_CONFIG(32); break;
       }
-#undef CG_GROUPED
+#undef CG_LANE_CONFIG
       return cudaGetLastError();
     }
-    uint64_t blocks = (total + per_block - 1) / per_block;
+    uint64_t blocks = (total + kRankThreads - 1) / kRankThreads;
     if (blocks > cap) blocks = cap;
-#define CG_GROUPED_CANARY(GG)                                                              \
-  auroc_grouped_canary_kernel<GG><<<(unsigned)blocks, kRankThreads, 0, stream>>>(           \
-      scores, labels, total, S, u2, gt, eq, status)
-    switch (G) {
-      case 2: CG_GROUPED_CANARY(2); break;
-      case 4: CG_GROUPED_CANARY(4); break;
-      case 8: CG_GROUPED_CANARY(8); break;
-      case 16: CG_GROUPED_CANARY(16); break;
-      default: CG_GROUPED_CANARY(32); break;
+#define CG_LANE_CANARY(P)                                                                   \
+  auroc_lane_canary_kernel<P><<<(unsigned)blocks, kRankThreads, 0, stream>>>(scores, labels, \
+                                                                           total, S, vec, u2, \
+                                                                           gt, eq, status)
+    switch (SP) {
+      case 4: CG_LANE_CANARY(4); break;
+      case 8: CG_LANE_CANARY(8); break;
+      case 16: CG_LANE_CANARY(16); break;
+      default: CG_LANE_CANARY(32); break;
     }
-#undef CG_GROUPED_CANARY
+#undef CG_LANE_CANARY
   }
   cudaError_t err = cudaGetLastError();
   if (err != cudaSuccess) return err;
