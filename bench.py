@@ -261,7 +261,9 @@ def oracle_describe(sample, passes, seconds):
 
 
 def oracle_baseline(cfg, n_threads, seconds):
-    """Time the oracle on the sample, repeating passes until `seconds` elapse."""
+    """Time the oracle on the sample, repeating passes until `seconds` elapse
+    on all `n_threads` cores; then one pass over a one-canary slice of the
+    sample on a single core."""
     sample = oracle_prepare(cfg, n_threads)
     elems = sample["S"] * sample["n"] * sample["L"]
     passes, t0 = 0, time.perf_counter()
@@ -271,8 +273,17 @@ def oracle_baseline(cfg, n_threads, seconds):
         el = time.perf_counter() - t0
         if el >= seconds:
             break
+    one = {"acts": np.ascontiguousarray(sample["acts"][:, :1]),
+           "refs": np.ascontiguousarray(sample["refs"][:, :1]),
+           "labels": np.ascontiguousarray(sample["labels"][:1]), "S": sample["S"], "n": 1,
+           "L": sample["L"]}
+    t1 = time.perf_counter()
+    oracle_pass(one, 1)
+    el1 = time.perf_counter() - t1
     return {"value": elems * passes / el, "unit": "elements/s", "cores": n_threads,
-            "kind": "oracle", "sample": oracle_describe(sample, passes, el)}
+            "kind": "oracle", "sample": oracle_describe(sample, passes, el),
+            "single_core": {"value": one["S"] * one["L"] / el1, "unit": "elements/s",
+                            "sample": oracle_describe(one, 1, el1)}}
 
 
 def run_reference(args, ranks: Ranks):

@@ -7,6 +7,18 @@
 
 #include "cg_internal.h"
 
+#include <nvtx3/nvToolsExt.h>
+
+// An NVTX range around every public call (visible in Nsight timelines; a
+// no-op unless a tool is attached).
+namespace {
+struct NvtxRange {
+  explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
+#define CG_TRACE(name) NvtxRange cg_nvtx_range_(name)
+
 static_assert(CG_NOALLOC_MAX_WORK_ITEMS == cg::kNoallocDriftItems,
               "public limit and scratch size disagree");
 static_assert(CG_NOALLOC_CHUNK_ELEMENTS == cg::kDriftChunk, "public chunk and kernel chunk disagree");
@@ -141,6 +153,7 @@ int cg_abi_version(void) { return 1; }
 cg_status cg_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
                           uint32_t first_block, uint32_t n_blocks, uint32_t *d_out,
                           cg_stream_t stream) {
+  CG_TRACE("cg_philox_words");
   if (!d_out || n_blocks == 0) return CG_ERR_INVALID_ARG;
   if (!aligned(d_out, 16)) return CG_ERR_ALIGNMENT;
   return from_cuda(cg::launch_philox_words(seed, c1, c2, c3, first_block, n_blocks, d_out,
@@ -150,6 +163,7 @@ cg_status cg_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
 cg_status cg_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
                             uint32_t first_block, uint32_t n_blocks, float *d_out,
                             cg_stream_t stream) {
+  CG_TRACE("cg_philox_normals");
   if (!d_out || n_blocks == 0) return CG_ERR_INVALID_ARG;
   if (!aligned(d_out, 16)) return CG_ERR_ALIGNMENT;
   return from_cuda(cg::launch_philox_normals(seed, c1, c2, c3, first_block, n_blocks, d_out,
@@ -167,6 +181,7 @@ cg_status cg_generate_workspace_size(const cg_pipeline_desc *desc, size_t *bytes
 cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts, float *d_refs,
                                int8_t *d_labels, void *d_ws, size_t ws_bytes, int32_t *d_status,
                                cg_stream_t stream) {
+  CG_TRACE("cg_generate_pipeline");
   cg_status st = check_desc(desc);
   if (st != CG_OK) return st;
   if (!d_acts || !d_refs) return CG_ERR_INVALID_ARG;
@@ -184,6 +199,7 @@ cg_status cg_generate_pipeline(const cg_pipeline_desc *desc, uint16_t *d_acts, f
 cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica, float *d_out,
                                 void *d_ws, size_t ws_bytes, int32_t *d_status,
                                 cg_stream_t stream) {
+  CG_TRACE("cg_generate_recompute");
   cg_status st = check_desc(desc);
   if (st != CG_OK) return st;
   if (!d_out) return CG_ERR_INVALID_ARG;
@@ -202,6 +218,7 @@ cg_status cg_generate_recompute(const cg_pipeline_desc *desc, uint32_t replica, 
 cg_status cg_generate_propagating(const cg_pipeline_desc *desc, float gain, uint16_t *d_acts,
                                   float *d_refs, int8_t *d_labels, void *d_ws, size_t ws_bytes,
                                   int32_t *d_status, cg_stream_t stream) {
+  CG_TRACE("cg_generate_propagating");
   cg_status st = check_desc(desc);
   if (st != CG_OK) return st;
   if (!isfinite(gain)) return CG_ERR_INVALID_ARG;
@@ -219,6 +236,7 @@ cg_status cg_generate_propagating(const cg_pipeline_desc *desc, float gain, uint
 cg_status cg_random_scores(uint64_t seed, uint32_t config_id0, uint32_t n_configs,
                            uint32_t n_canaries, uint32_t n_shards, float *d_scores,
                            cg_stream_t stream) {
+  CG_TRACE("cg_random_scores");
   if (!d_scores || n_configs == 0 || n_canaries == 0 || n_shards == 0) return CG_ERR_INVALID_ARG;
   if ((uint64_t)config_id0 + n_configs > (1ull << 30)) return CG_ERR_INVALID_ARG;
   if (n_canaries > (1u << 24)) return CG_ERR_UNSUPPORTED;
@@ -247,6 +265,7 @@ cg_status cg_drift_scores_ex(const uint16_t *d_acts, const float *d_refs, uint32
                              uint32_t n_canaries, uint64_t seg_len, float *d_scores,
                              uint64_t stat_stride, void *d_ws, size_t ws_bytes, int32_t *d_status,
                              int32_t algo, cg_stream_t stream) {
+  CG_TRACE("cg_drift_scores_ex");
   if (!d_acts || !d_refs || !d_scores || n_shards == 0 || n_canaries == 0 || seg_len == 0)
     return CG_ERR_INVALID_ARG;
   if (algo < CG_DRIFT_AUTO || algo > CG_DRIFT_BULK_2CTA) return CG_ERR_INVALID_ARG;
@@ -274,6 +293,7 @@ cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs, uint
                                uint32_t n_canaries, uint64_t seg_len, float *d_scores,
                                uint64_t stat_stride, void *d_ws, size_t ws_bytes,
                                int32_t *d_status, cg_stream_t stream) {
+  CG_TRACE("cg_drift_scores_host");
   if (!h_acts) return CG_ERR_INVALID_ARG;
   // Only page-locked host memory registered with CUDA may be read by a
   // kernel; resolve its device-side address (equal to the host address
@@ -293,6 +313,7 @@ cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,
                                   uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
                                   float *d_scores, uint64_t stat_stride, int32_t *d_status,
                                   cg_stream_t stream) {
+  CG_TRACE("cg_drift_scores_noalloc");
   if (n_shards == 0 || n_canaries == 0 || seg_len == 0) return CG_ERR_INVALID_ARG;
   const uint64_t n_seg = (uint64_t)n_shards * n_canaries;
   if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
@@ -312,6 +333,7 @@ cg_status cg_make_control_labels(const int8_t *d_labels, uint32_t n_configs,
                                  uint32_t n_canaries, uint32_t n_shards, uint64_t seed,
                                  uint32_t config_id0, int8_t *d_ctrl, int32_t *d_status,
                                  cg_stream_t stream) {
+  CG_TRACE("cg_make_control_labels");
   if (!d_labels || !d_ctrl || n_configs == 0 || n_canaries == 0 || n_shards == 0)
     return CG_ERR_INVALID_ARG;
   if ((uint64_t)config_id0 + n_configs > (1ull << 30)) return CG_ERR_INVALID_ARG;
@@ -326,6 +348,7 @@ cg_status cg_make_control_labels(const int8_t *d_labels, uint32_t n_configs,
 cg_status cg_auroc(const float *d_scores, const int8_t *d_labels, uint32_t n_configs,
                    uint32_t n_canaries, uint32_t n_shards, int64_t *d_u2, int64_t *d_gt,
                    int64_t *d_eq, double *d_auroc, int32_t *d_status, cg_stream_t stream) {
+  CG_TRACE("cg_auroc");
   if (!d_scores || !d_labels || !d_u2 || !d_auroc || n_configs == 0 || n_canaries == 0 ||
       n_shards == 0)
     return CG_ERR_INVALID_ARG;
@@ -343,6 +366,7 @@ cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels, uint32_
                           uint32_t n_canaries, uint32_t n_shards, int64_t *d_u2,
                           int64_t *d_n_mal, int64_t *d_n_ben, double *d_auroc, int32_t *d_status,
                           cg_stream_t stream) {
+  CG_TRACE("cg_auroc_pooled");
   if (!d_scores || !d_labels || !d_u2 || !d_auroc || n_configs == 0 || n_canaries == 0 ||
       n_shards == 0)
     return CG_ERR_INVALID_ARG;
@@ -358,12 +382,14 @@ cg_status cg_auroc_pooled(const float *d_scores, const int8_t *d_labels, uint32_
 }
 
 cg_status cg_selftest_bounded_wait(uint32_t limit_us, int32_t *d_status, cg_stream_t stream) {
+  CG_TRACE("cg_selftest_bounded_wait");
   if (!d_status || limit_us == 0 || limit_us > 10u * 1000u * 1000u) return CG_ERR_INVALID_ARG;
   if (!aligned(d_status, 4)) return CG_ERR_ALIGNMENT;
   return from_cuda(cg::launch_bounded_wait_probe(limit_us, d_status, (cudaStream_t)stream));
 }
 
 cg_status cg_read_status(const int32_t *d_status, cg_stream_t stream, int32_t *h_word) {
+  CG_TRACE("cg_read_status");
   if (!d_status) return CG_ERR_INVALID_ARG;
   int32_t w = 0;
   cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
