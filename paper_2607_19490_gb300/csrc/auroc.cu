@@ -212,21 +212,28 @@ __device__ __forceinline__ void lane_counts(const float *__restrict__ scores,
       l[k] = (uint32_t)k < S ? (int)ls[k] : -1;
     }
   }
-  int lg = 0, le = 0, cm = 0, cb = 0;
+  // stage bitmasks; only the malicious stages are walked, the benign
+  // comparison is unrolled (m_i picked by selects, no dynamic indexing)
+  uint32_t mal = 0u, ben = 0u;
 #pragma unroll
-  for (int i = 0; i < SP; ++i) {
-    if ((l[i] == 0 || l[i] == 1) && is_nan_f(m[i])) saw_nan = true;
-    cm += (l[i] == 1);
-    cb += (l[i] == 0);
+  for (int k = 0; k < SP; ++k) {
+    if ((l[k] == 0 || l[k] == 1) && is_nan_f(m[k])) saw_nan = true;
+    mal |= (uint32_t)(l[k] == 1) << k;
+    ben |= (uint32_t)(l[k] == 0) << k;
   }
+  const int cm = __popc(mal), cb = __popc(ben);
+  int lg = 0, le = 0;
+  while (mal) {
+    const int i = __ffs(mal) - 1;
+    mal &= mal - 1u;
+    float mi = 0.f;
 #pragma unroll
-  for (int i = 0; i < SP; ++i) {
-    if (l[i] != 1) continue;
+    for (int k = 0; k < SP; ++k) mi = (k == i) ? m[k] : mi;
 #pragma unroll
     for (int j = 0; j < SP; ++j) {
-      const bool b = l[j] == 0;
-      lg += (b && m[i] > m[j]);
-      le += (b && m[i] == m[j]);
+      const bool b = (ben >> j) & 1u;
+      lg += (b && mi > m[j]);
+      le += (b && mi == m[j]);
     }
   }
   g = lg;

@@ -444,22 +444,6 @@ drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ r
 
 }  // namespace
 
-// Diagnostic for the bounded wait: one warp waits on a phase of an mbarrier
-// that nothing arrives at.  The wait must give up after limit_ns and raise
-// CG_DEVFLAG_TIMEOUT; no copy is in flight, so the block can leave.
-__global__ void bounded_wait_probe_kernel(unsigned long long limit_ns, int32_t *status) {
-  __shared__ __align__(8) unsigned long long bar;
-  const uint32_t b = (uint32_t)__cvta_generic_to_shared(&bar);
-  if (threadIdx.x == 0) {
-    mbar_init(b, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  __syncthreads();
-  const bool done = mbar_wait(b, 0u, limit_ns);
-  if (!__all_sync(0xFFFFFFFFu, done) && threadIdx.x == 0 && status)
-    atomicOr(status, CG_DEVFLAG_TIMEOUT);
-}
-
 template <int NS>
 static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t seg_len,
                                uint64_t cps, uint64_t n_items, float4 *partials, int32_t *status,
@@ -478,6 +462,22 @@ static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t
   drift_bulk_kernel<NS><<<(unsigned)grid, kBulkThreads, smem, stream>>>(acts, refs, seg_len, cps,
                                                                         n_items, partials, status);
   return cudaGetLastError();
+}
+
+// Diagnostic for the bounded wait: one warp waits on a phase of an mbarrier
+// that nothing arrives at.  The wait must give up after limit_ns and raise
+// CG_DEVFLAG_TIMEOUT; no copy is in flight, so the block can leave.
+__global__ void bounded_wait_probe_kernel(unsigned long long limit_ns, int32_t *status) {
+  __shared__ __align__(8) unsigned long long bar;
+  const uint32_t b = (uint32_t)__cvta_generic_to_shared(&bar);
+  if (threadIdx.x == 0) {
+    mbar_init(b, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const bool done = mbar_wait(b, 0u, limit_ns);
+  if (!__all_sync(0xFFFFFFFFu, done) && threadIdx.x == 0 && status)
+    atomicOr(status, CG_DEVFLAG_TIMEOUT);
 }
 
 bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len) {
