@@ -698,14 +698,14 @@ def launches_per_config(cfg) -> int:
     return gen + 2 + 1 + 4 * 2 + 1
 
 
-def study_oracle_baseline(configs, seconds):
+def study_oracle_baseline(cfgs, seconds):
     """The fp64 oracle on a bounded sample of the study: its configurations in
     order, each with its canaries cut to at most 8, until `seconds` pass."""
     from oracle import oracle as O
     O.build()
     threads = O.max_threads()
     done, t0 = 0, time.perf_counter()
-    for cfg in configs:
+    for cfg in cfgs:
         sub = SI.shrink(cfg, n_canaries=min(8, cfg["n_canaries"]))
         gain = sub.pop("gain", 0.0)
         D = O.desc_from_dict(sub)
@@ -720,8 +720,9 @@ def study_oracle_baseline(configs, seconds):
         if time.perf_counter() - t0 >= seconds:
             break
     el = time.perf_counter() - t0
-    frac = min(8, configs[0]["n_canaries"]) / configs[0]["n_canaries"]
-    return {"value": done * frac / el, "unit": "configs/s", "cores": threads, "kind": "oracle",
+    first = cfgs[0] if cfgs else {"n_canaries": 1}
+    frac = min(8, first["n_canaries"]) / first["n_canaries"]
+    return {"value": done * frac / el, "unit": "cfgs/s", "cores": threads, "kind": "oracle",
             "sample": f"first {done} configurations with at most 8 canaries each (generate + "
                       f"drift + AUROC in fp64), scaled to full canary counts by {frac:.3f}, "
                       f"{el:.1f} s"}
