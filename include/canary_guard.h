@@ -216,7 +216,7 @@ typedef enum {
   CG_DRIFT_AUTO = 0,       /* CG_DRIFT_BULK when both inputs are device memory and
                               seg_len % 8 == 0, else CG_DRIFT_STREAM (cg_drift_scores) */
   CG_DRIFT_STREAM = 1,     /* register-streaming kernel, any seg_len */
-  CG_DRIFT_BULK = 2,       /* TMA bulk-copy pipeline, 8 shared-memory stages, 1 block per SM;
+  CG_DRIFT_BULK = 2,       /* TMA bulk-copy pipeline, 6 shared-memory stages, 1 block per SM;
                               needs device memory and seg_len % 8 == 0
                               (else CG_ERR_UNSUPPORTED) */
   CG_DRIFT_BULK_2CTA = 3   /* TMA bulk-copy pipeline, 4 stages, 2 blocks per SM; same need */

@@ -495,7 +495,7 @@ cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t 
   float4 *partials = reinterpret_cast<float4 *>(static_cast<char *>(ws) + kDriftHeader);
   cudaError_t err;
   if (algo == CG_DRIFT_BULK) {
-    err = launch_bulk<8>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
+    err = launch_bulk<6>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
   } else if (algo == CG_DRIFT_BULK_2CTA) {
     err = launch_bulk<4>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
   } else {
