@@ -576,7 +576,7 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
 STUDY_METRIC = "AUROC configs/sec (whole study: generate, score and rank every configuration)"
 
 
-def study_pass(cg, torch, configs, dev, bufs, res):
+def study_pass(cg, torch, configs, dev, bufs, res, drift_events=None):
     """Every configuration of a study on the device: generate, drift scores,
     control labels, per-canary AUROC of rel_l2 / max_abs / cos_dev and of the
     control, pooled AUROC of rel_l2.  res[c] = those five A-hat values."""
@@ -595,7 +595,11 @@ def study_pass(cg, torch, configs, dev, bufs, res):
             cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"],
                                     status=bufs["status"])
         scores = bufs["scores"][:3 * N * S].view(3, N, S)
+        if drift_events is not None:
+            drift_events[c][0].record()
         cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"], status=bufs["status"])
+        if drift_events is not None:
+            drift_events[c][1].record()
         cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
                                   status=bufs["status"])
         u2 = bufs["u2"][:N].view(1, N)
@@ -657,6 +661,15 @@ def run_study(args, ranks: Ranks):
     st, word = cg.cg_read_status(bufs["status"])
     if st != 0:
         raise RuntimeError(f"device status {word} during the study")
+    # one more pass with events around every drift call: the drift reduction's
+    # own bandwidth on these pipelines (6 algorithmic bytes per element)
+    dev_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in configs]
+    study_pass(cg, torch, configs, dev, bufs, res, drift_events=dev_ev)
+    torch.cuda.synchronize()
+    drift_ms = sum(a.elapsed_time(b) for a, b in dev_ev)
+    drift_bytes = float(sum(SI.n_elements(c) for c in configs)) * BYTES_PER_ELEMENT
+    peak, peak_kind = measured_peaks()
     A = res.cpu().numpy()
     total_cfg = ranks.sum(float(len(configs)))
     elems = ranks.sum(float(sum(SI.n_elements(c) for c in configs)))
@@ -680,6 +693,10 @@ def run_study(args, ranks: Ranks):
                    "step": "per configuration: generate (4 kernels), drift (2), control labels, "
                            "3 + 1 per-canary AUROC, 1 pooled AUROC"},
         "elements_per_s": elems / (ms / 1e3),
+        "drift": {"ms_per_pass": drift_ms, "GBps": drift_bytes / (drift_ms / 1e3) / 1e9,
+                  "frac": drift_bytes / (drift_ms / 1e3) / 1e9 / peak,
+                  "peak_GBps": peak, "peak_kind": f"{peak_kind} copy bandwidth",
+                  "elements_per_s": drift_bytes / BYTES_PER_ELEMENT / (drift_ms / 1e3)},
         "auroc_summary": summary,
         "per_config_auroc": {n: [round(float(x), 6) for x in A[:, k]] for k, n in enumerate(names)},
         "cpu_baseline": cpu,

@@ -98,3 +98,33 @@ def test_matches_oracle_when_decisive(cg, orc, study, idx):
         assert g == o
     else:
         assert abs(g - o) <= 0.1
+
+
+@pytest.mark.parametrize("study,idx", [("factorial", 323), ("factorial", 300), ("factorial", 270),
+                                       ("snr", 6), ("snr", 0)])
+def test_full_size_configs_sampled_against_oracle(cg, orc, study, idx):
+    """The largest factorial configurations (16 x 8192 x 64 x 64) and the
+    noise-floor steps (8 x 4096 x 128 x 128) at full size: sampled segments of
+    the generator against the oracle, and neutral bytes planted into sampled
+    segments scored in the same launch as the rest of the pipeline."""
+    import torch
+    from tests._cmp import assert_normals_close, assert_scores_close, half_ulp_distance
+    cfg = SI.STUDIES[study]()[idx]
+    S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
+    acts, refs, labels = cg.cg_generate_pipeline(cg.PipelineDesc.from_config(cfg))
+    D = orc.desc_from_dict(cfg)
+    picks = [(0, 0), (cfg["malicious"][0], N - 1), (S // 2, N // 2)]
+    for s, n in picks:
+        o_r, _, o_a, _ = orc.generate_segment(D, s, n)
+        assert_normals_close(refs[s, n].cpu().numpy(), o_r, what="references")
+        assert half_ulp_distance(acts[s, n].cpu().numpy().view(np.uint16), o_a).max() <= 1
+    planted = {}
+    for i, (s, n) in enumerate([(1, 1), (S - 1, 0)]):
+        pa, pr = SI.drift_arrays(1, 1, L, seed=900 + i)
+        acts[s, n].copy_(torch.from_numpy(pa.view(np.float16).reshape(-1)))
+        refs[s, n].copy_(torch.from_numpy(pr.reshape(-1)))
+        planted[(s, n)] = (pa.reshape(-1), pr.reshape(-1))
+    scores = cg.cg_drift_scores(acts, refs, S, N).cpu().numpy()
+    for (s, n), (pa, pr) in planted.items():
+        out, _ = orc.drift_segment(pa, pr)
+        assert_scores_close(scores[:, n, s][:, None], out[:, None], what=f"segment {(s, n)}")
