@@ -122,6 +122,15 @@ cg::GenParams make_params(const cg_pipeline_desc &d, const cg::GenLayout &lay) {
   p.n_flip = nf;
   p.mask_words = lay.mask_words;
   p.stat_chunks = lay.stat_chunks;
+  {
+    uint32_t k0 = (uint32_t)d.seed, k1 = (uint32_t)(d.seed >> 32);
+    for (int r = 0; r < 10; ++r) {   // Philox round keys (SC'11 key schedule)
+      p.round_keys[2 * r] = k0;
+      p.round_keys[2 * r + 1] = k1;
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+  }
   for (uint32_t i = 0; i < d.n_malicious; ++i) {
     const uint32_t s = (uint32_t)d.malicious[i];
     p.mal_bits[s >> 5] |= 1u << (s & 31);

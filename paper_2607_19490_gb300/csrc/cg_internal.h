@@ -74,6 +74,7 @@ struct GenParams {
   uint32_t n_outlier, n_flip;   // flipped channels per malicious stage
   uint32_t mask_words;
   uint64_t stat_chunks;
+  uint32_t round_keys[20];      // Philox round keys of `seed` (key + r * Weyl constants)
   int32_t recompute;            // 1: write a benign recompute of every stage into refs
   uint32_t noise_c3;            // counter word 3 of the noise stream (recompute replica)
   uint32_t mal_bits[kMaxShards / 32];

@@ -36,6 +36,24 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
   return c;
 }
 
+// The ten round keys of one seed, (key + r W0, key + r W1) for r = 0..9.
+// They are the same for every draw of a launch, so the generator kernels take
+// them precomputed (kernel parameters) and each round folds its key into the
+// XOR instead of advancing it.
+struct PhiloxRoundKeys {
+  uint32_t k[20];
+};
+
+__device__ __forceinline__ uint4 philox4x32_10_rk(uint4 c, const PhiloxRoundKeys &rk) {
+#pragma unroll
+  for (int round = 0; round < 10; ++round) {
+    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
+    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
+    c = make_uint4(hi1 ^ c.y ^ rk.k[2 * round], lo1, hi0 ^ c.w ^ rk.k[2 * round + 1], lo0);
+  }
+  return c;
+}
+
 __device__ __forceinline__ uint2 philox_key(uint64_t seed) {
   return make_uint2((uint32_t)seed, (uint32_t)(seed >> 32));
 }
@@ -50,6 +68,15 @@ __device__ __forceinline__ float2 box_muller(uint32_t x0, uint32_t x1) {
   float s, c;
   sincospif(2.0f * u2, &s, &c);
   return make_float2(r * c, r * s);
+}
+
+// The four normals of one Philox block from precomputed round keys.
+__device__ __forceinline__ float4 normals4_rk(const PhiloxRoundKeys &rk, uint32_t q, uint32_t c1,
+                                              uint32_t c2, uint32_t c3 = 0u) {
+  const uint4 w = philox4x32_10_rk(make_uint4(q, c1, c2, c3), rk);
+  const float2 a = box_muller(w.x, w.y);
+  const float2 b = box_muller(w.z, w.w);
+  return make_float4(a.x, a.y, b.x, b.y);
 }
 
 // The four normals of one Philox block (counter word 3 = c3: 0 for every

@@ -449,14 +449,29 @@ static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t
                                uint64_t cps, uint64_t n_items, float4 *partials, int32_t *status,
                                int sm_count, cudaStream_t stream) {
   const size_t smem = sizeof(BulkSmem<NS>);
-  cudaError_t err = cudaFuncSetAttribute(drift_bulk_kernel<NS>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  // shared-memory opt-in and occupancy, once per device
+  static std::mutex mu;
+  static int per_sm_of[64] = {};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  int per_sm = 0;
-  err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, drift_bulk_kernel<NS>, kBulkThreads,
-                                                      smem);
-  if (err != cudaSuccess) return err;
-  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  int per_sm;
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (per_sm_of[dev] == 0) {
+      err = cudaFuncSetAttribute(drift_bulk_kernel<NS>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (err != cudaSuccess) return err;
+      int n = 0;
+      err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, drift_bulk_kernel<NS>, kBulkThreads,
+                                                          smem);
+      if (err != cudaSuccess) return err;
+      if (n < 1) return cudaErrorInvalidConfiguration;
+      per_sm_of[dev] = n;
+    }
+    per_sm = per_sm_of[dev];
+  }
   uint64_t grid = (uint64_t)sm_count * (uint64_t)per_sm;
   if (grid > n_items) grid = n_items;
   drift_bulk_kernel<NS><<<(unsigned)grid, kBulkThreads, smem, stream>>>(acts, refs, seg_len, cps,

@@ -103,12 +103,12 @@ __device__ __forceinline__ float ref_value(float z, uint32_t c, const GenParams 
 // need: sum |a| on a benign stage under the Eq. 2 model (mu = ||a||_1 / (T d));
 // sum a^2 and the tamper direction's sum g^2 on a Gaussian-tamper stage
 // (tau(v) = v + eps ||v|| g / ||g||).  One double2 per item.
-__device__ __forceinline__ void normals8(uint2 key, uint32_t q0, uint32_t seg, uint32_t c2,
-                                         uint32_t c3, int cnt, float z[8]) {
-  const float4 a = normals4(key, q0, seg, c2, c3);
+__device__ __forceinline__ void normals8(const PhiloxRoundKeys &rk, uint32_t q0, uint32_t seg,
+                                         uint32_t c2, uint32_t c3, int cnt, float z[8]) {
+  const float4 a = normals4_rk(rk, q0, seg, c2, c3);
   z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
   if (cnt > 4) {
-    const float4 b = normals4(key, q0 + 1, seg, c2, c3);
+    const float4 b = normals4_rk(rk, q0 + 1, seg, c2, c3);
     z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
   } else {
     z[4] = z[5] = z[6] = z[7] = 0.f;
@@ -120,7 +120,7 @@ gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *_
                 double2 *__restrict__ stats) {
   __shared__ double2 warp_sum[kGenThreads / 32];
   const uint64_t n_items = (uint64_t)p.S * p.N * p.stat_chunks;
-  const uint2 key = philox_key(p.seed);
+  const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_ref = 4u * p.config_id + kStreamRef;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   const int tid = threadIdx.x;
@@ -137,7 +137,7 @@ gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *_
     for (uint64_t e0 = e_begin + 8 * (uint64_t)tid; e0 < e_end; e0 += 8 * (uint64_t)kGenThreads) {
       const int cnt = (int)min((uint64_t)8, p.L - e0);
       float z[8], a[8];
-      normals8(key, (uint32_t)(e0 >> 2), seg, c2_ref, 0u, cnt, z);
+      normals8(rk, (uint32_t)(e0 >> 2), seg, c2_ref, 0u, cnt, z);
       uint32_t c = (uint32_t)(e0 % p.d);
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
@@ -148,7 +148,7 @@ gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *_
         for (int k = 0; k < cnt; ++k) x += fabsf(a[k]);
       } else if (need_l2) {
         float g[8];
-        normals8(key, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, g);
+        normals8(rk, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, g);
         for (int k = 0; k < cnt; ++k) {
           x = fmaf(a[k], a[k], x);
           y = fmaf(g[k], g[k], y);
@@ -222,7 +222,7 @@ gen_live_kernel(GenParams p, const uint32_t *__restrict__ flip_mask, const float
                 uint16_t *__restrict__ acts, float *__restrict__ refs) {
   const uint64_t groups_per_seg = (p.L + 7) >> 3;
   const uint64_t total = (uint64_t)p.S * p.N * groups_per_seg;
-  const uint2 key = philox_key(p.seed);
+  const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   for (uint64_t gi = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < total;
@@ -251,7 +251,7 @@ gen_live_kernel(GenParams p, const uint32_t *__restrict__ flip_mask, const float
     const float cf = coef[seg];
     if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
       float n[8];
-      normals8(key, q0, seg, mal ? c2_tamper : c2_noise, mal ? 0u : p.noise_c3, cnt, n);
+      normals8(rk, q0, seg, mal ? c2_tamper : c2_noise, mal ? 0u : p.noise_c3, cnt, n);
       if (!mal && p.noise == CG_NOISE_MULT) {
 #pragma unroll
         for (int k = 0; k < 8; ++k) h[k] = a[k] * (1.0f + cf * n[k]);   // a (1 + sigma_s z)
@@ -359,7 +359,7 @@ gen_prop_stats_kernel(GenParams p, uint32_t s, float gain, const float *__restri
                       const uint16_t *__restrict__ acts, double2 *__restrict__ stats) {
   __shared__ double2 warp_sum[kGenThreads / 32];
   const uint64_t n_items = (uint64_t)p.N * p.stat_chunks;
-  const uint2 key = philox_key(p.seed);
+  const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   const bool mal = is_malicious(p, s);
   const bool need_l1 = !mal && p.noise == CG_NOISE_PAPER;
@@ -385,7 +385,7 @@ gen_prop_stats_kernel(GenParams p, uint32_t s, float gain, const float *__restri
           for (int k = 0; k < cnt; ++k) x += fabsf(v[k]);
         } else {
           float gg[8];
-          normals8(key, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, gg);
+          normals8(rk, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, gg);
           for (int k = 0; k < cnt; ++k) {
             x = fmaf(v[k], v[k], x);
             y = fmaf(gg[k], gg[k], y);
@@ -419,7 +419,7 @@ gen_prop_live_kernel(GenParams p, uint32_t s, float gain, const uint32_t *__rest
                      uint16_t *__restrict__ acts) {
   const uint64_t groups_per_seg = (p.L + 7) >> 3;
   const uint64_t total = (uint64_t)p.N * groups_per_seg;
-  const uint2 key = philox_key(p.seed);
+  const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
   const bool mal = is_malicious(p, s);
@@ -439,7 +439,7 @@ gen_prop_live_kernel(GenParams p, uint32_t s, float gain, const uint32_t *__rest
     const float cf = coef[seg];
     if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
       float z[8];
-      normals8(key, q0, seg, mal ? c2_tamper : c2_noise, 0u, cnt, z);
+      normals8(rk, q0, seg, mal ? c2_tamper : c2_noise, 0u, cnt, z);
       if (!mal && p.noise == CG_NOISE_MULT) {
 #pragma unroll
         for (int k = 0; k < 8; ++k) h[k] = v[k] * (1.0f + cf * z[k]);
