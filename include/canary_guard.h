@@ -202,7 +202,9 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * seg_len >= 1 (ragged tails handled).  Scores are written to
  * d_scores[stat * stat_stride + n * S + s] (stat_stride >= N * S; pass
  * N * S for a dense [3][N][S] block).  Each element of d_acts and d_refs is
- * read once from HBM.  d_ws: >= cg_drift_workspace_size bytes, 16-byte
+ * read once from HBM.  Sums are accumulated in fp32 per chunk of 16384
+ * elements and combined in fp64, so element magnitudes must stay below
+ * about 1e17 for the squared sums to remain finite.  d_ws: >= cg_drift_workspace_size bytes, 16-byte
  * aligned, scratch.
  */
 cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
