@@ -555,6 +555,24 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
            "inputs": "live fp16 activations read from pinned host memory every step by "
                      "cg_drift_scores_host; fp32 references resident in HBM"}
 
+    # the same step with an explicit copy-engine transfer of the live
+    # activations (cudaMemcpyAsync into device memory) before the drift pass
+    def step_copy(i):
+        acts.copy_(h_acts, non_blocking=True)
+        cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=dws)
+        cg.cg_make_control_labels(labels, seed=5000 + i, ctrl=ctrl)
+        cg.cg_auroc(scores[0][None], labels, auroc=auroc[0:1], want_counts=False)
+        cg.cg_auroc(scores[0][None], ctrl, auroc=auroc[1:2], want_counts=False)
+        h_scores.copy_(scores, non_blocking=True)
+        h_auroc.copy_(auroc, non_blocking=True)
+
+    ms_copy = timed(step_copy, args.e2e_steps)
+    out["memcpy_variant"] = {"value": elems / (ms_copy / 1e3), "unit": "elements/s",
+                             "h2d_bytes_per_step": h2d, "ms_per_step": ms_copy,
+                             "link_GBps": h2d / (ms_copy / 1e3) / 1e9,
+                             "inputs": "live activations copied with cudaMemcpyAsync, then the "
+                                       "device-resident drift pass"}
+
     h_refs = torch.empty(refs.shape, dtype=refs.dtype, pin_memory=True)
     h_refs.copy_(refs)
 
