@@ -35,9 +35,6 @@ inline size_t drift_ws_bytes(uint64_t n_segments, uint64_t seg_len) {
   return kDriftHeader + align_up((size_t)(n_segments * drift_chunks_per_seg(seg_len)) * 16, 256);
 }
 
-cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
-                         uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
-                         cudaStream_t stream);
 
 cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream);
 bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len);

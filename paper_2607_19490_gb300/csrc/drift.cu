@@ -3,18 +3,23 @@
 // verifier: every fp16 live element and every fp32 reference element is
 // read exactly once (6 bytes per element).
 //
-// Pass 1 (drift_partial_kernel): the [S][N][L] element space is cut into
-// work items of at most kDriftChunk elements, never crossing a segment.  A
-// persistent grid (SM count x resident blocks) walks the items in order.
-// Each thread streams 16-byte vectors (8 fp16 live values, 2 x 4 fp32
-// references) with non-allocating, 256-byte-prefetching global loads, four
-// vectors in flight, and accumulates in fp32:
+// Pass 1 cuts the [S][N][L] element space into work items of at most
+// kDriftChunk elements, never crossing a segment, and writes one float4 of
+// fp32 sums per item:
 //     D = sum (h - a)^2,   E = sum (h - a)(h + a) = sum h^2 - a^2,
 //     A = sum a^2,         M = max |h - a|
-// The block reduces its sums with warp shuffles and a fixed tree and writes
-// one float4 per item.  Pass 2 (drift_finalize_kernel) combines the items of
-// a segment in order in fp64 and writes the three scores.  No atomics, so
-// the result is the same on every run.
+// by one of two kernels:
+//   drift_bulk_kernel     (default for device memory, seg_len % 8 == 0) a TMA
+//                         pipeline: one producer warp fills a shared-memory
+//                         ring with cp.async.bulk copies tracked by mbarriers,
+//                         eight consumer warps accumulate;
+//   drift_partial_kernel  (any seg_len, host-resident input, the no-alloc
+//                         entry point) a persistent grid whose threads keep
+//                         four 16-byte vectors per stream in flight with
+//                         non-allocating, 256-byte-prefetching loads.
+// Pass 2 (drift_finalize_kernel) combines the items of a segment in a fixed
+// order in fp64 and writes the three scores.  No atomics, so the result is
+// the same on every run.
 #include <cuda_fp16.h>
 
 #include <mutex>
@@ -528,25 +533,6 @@ cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t 
 cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream) {
   bounded_wait_probe_kernel<<<1, 32, 0, stream>>>(1000ull * limit_us, status);
   return cudaGetLastError();
-}
-
-cudaError_t launch_drift(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
-                         uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
-                         cudaStream_t stream) {
-  DeviceInfo info;
-  if (!device_info(&info)) return cudaGetLastError();
-  const uint64_t n_seg = (uint64_t)S * N;
-  const uint64_t cps = drift_chunks_per_seg(seg_len);
-  const uint64_t n_items = n_seg * cps;
-  float4 *partials = reinterpret_cast<float4 *>(static_cast<char *>(ws) + kDriftHeader);
-  uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
-  if (grid > n_items) grid = n_items;
-  if (grid < 1) grid = 1;
-  drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
-                                                                     n_items, partials);
-  cudaError_t err = cudaGetLastError();
-  if (err != cudaSuccess) return err;
-  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
 }
 
 int drift_occupancy() {
