@@ -189,30 +189,33 @@ drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_s
     M = fmaxf(M, __shfl_down_sync(0xFFFFFFFFu, M, off));
   }
   if (lane != 0) return;
-  double rel, cosd;
+  // The sums stay fp64; the scores are formed in fp32 from them (GB300's
+  // FP64 pipe is narrow, and fp32 sqrt/div of the rounded sums is accurate
+  // to a few 1e-7 relative, far inside the drift tolerances).
+  float rel, cosd;
   if (isnan(D) || isnan(A)) {
     rel = NAN;
   } else if (A > 0.0) {
-    rel = sqrt(D / A);
+    rel = sqrtf((float)D / (float)A);
   } else {
-    rel = (D == 0.0) ? 0.0 : INFINITY;
+    rel = (D == 0.0) ? 0.f : INFINITY;
   }
   const double H = A + E;
   if (isnan(D) || isnan(E) || isnan(A)) {
     cosd = NAN;
   } else if (H > 0.0 && A > 0.0) {
-    const double sh = sqrt(H), sa = sqrt(A);
-    const double gap = E / (sh + sa);
-    cosd = (D - gap * gap) / (2.0 * sh * sa);
-    cosd = fmin(fmax(cosd, 0.0), 2.0);
+    const float sh = sqrtf((float)H), sa = sqrtf((float)A);
+    const float gap = (float)E / (sh + sa);
+    cosd = ((float)D - gap * gap) / (2.0f * sh * sa);
+    cosd = fminf(fmaxf(cosd, 0.f), 2.f);
   } else {
-    cosd = 0.0;
+    cosd = 0.f;
   }
   const uint32_t s = (uint32_t)(seg / N), n = (uint32_t)(seg % N);
   const uint64_t o = (uint64_t)n * S + s;
-  scores[o] = (float)rel;
+  scores[o] = rel;
   scores[stat_stride + o] = M;
-  scores[2 * stat_stride + o] = (float)cosd;
+  scores[2 * stat_stride + o] = cosd;
 }
 
 static cudaError_t launch_finalize(const float4 *partials, uint64_t cps, uint32_t S, uint32_t N,
