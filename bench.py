@@ -708,7 +708,7 @@ def run_study(args, ranks: Ranks):
         "data": "synthetic",
         "config": {"workload": f"study '{args.study}': {len(configs)} configurations",
                    "elements_per_pass": elems,
-                   "step": "per configuration: generate (4 kernels), drift (2), control labels, "
+                   "step": "per configuration: generate (2 to 4 kernels), drift (2), control labels, "
                            "3 + 1 per-canary AUROC, 1 pooled AUROC"},
         "elements_per_s": elems / (ms / 1e3),
         "drift": {"ms_per_pass": drift_ms, "GBps": drift_bytes / (drift_ms / 1e3) / 1e9,

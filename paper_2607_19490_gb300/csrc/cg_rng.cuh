@@ -47,9 +47,10 @@ struct PhiloxRoundKeys {
 __device__ __forceinline__ uint4 philox4x32_10_rk(uint4 c, const PhiloxRoundKeys &rk) {
 #pragma unroll
   for (int round = 0; round < 10; ++round) {
-    const uint32_t hi0 = __umulhi(kPhiloxM0, c.x), lo0 = kPhiloxM0 * c.x;
-    const uint32_t hi1 = __umulhi(kPhiloxM1, c.z), lo1 = kPhiloxM1 * c.z;
-    c = make_uint4(hi1 ^ c.y ^ rk.k[2 * round], lo1, hi0 ^ c.w ^ rk.k[2 * round + 1], lo0);
+    const uint64_t p0 = (uint64_t)kPhiloxM0 * c.x;   // one 32x32 -> 64 multiply each
+    const uint64_t p1 = (uint64_t)kPhiloxM1 * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ rk.k[2 * round], (uint32_t)p1,
+                   (uint32_t)(p0 >> 32) ^ c.w ^ rk.k[2 * round + 1], (uint32_t)p0);
   }
   return c;
 }

@@ -5,14 +5,18 @@
 //   gen_setup_kernel    per-configuration draws: outlier-channel mask,
 //                       per-stage sigma (lognormal spread), flipped-channel
 //                       masks of the malicious stages; labels [N][S]
-//   gen_refs_kernel     pass 1: reference normals -> fp32 references, plus
-//                       the per-chunk sums the live values depend on:
-//                       sum |a| (Eq. 2: mu = ||a||_1 / (T d)) for benign
-//                       stages under the Eq. 2 noise model; sum a^2 and
-//                       sum g^2 (the Gaussian tamper's ||v|| and ||g||)
+//   gen_refs_kernel     pass 1: reference normals -> fp32 references.  A
+//                       segment whose live values follow element by element
+//                       (benign a (1 + sigma_s z), sign flips, rescale) gets
+//                       its fp16 live values here too, from the registers.
+//                       The other segments get the sums their live values
+//                       depend on: sum |a| (Eq. 2: mu = ||a||_1 / (T d)) for
+//                       benign stages under the Eq. 2 noise model; sum a^2
+//                       and sum g^2 (the Gaussian tamper's ||v|| and ||g||)
 //   gen_coef_kernel     per-segment scalar from those sums (fixed order, fp64)
-//   gen_live_kernel     pass 2: references read back, noise or tamper
-//                       normals drawn, fp16 live values stored
+//   gen_live_kernel     pass 2, only for those segments: references read
+//                       back, noise or tamper normals drawn, fp16 live
+//                       values stored
 // Random draws follow the counter layout of cg_rng.cuh: element e of
 // segment seg on stream k uses block e / 4 of counter
 // (e / 4, seg, 4 config_id + k, 0).
@@ -88,21 +92,9 @@ __global__ void gen_setup_kernel(GenParams p, uint32_t *outlier_mask, uint32_t *
   if (gave_up && status) atomicOr(status, CG_DEVFLAG_TIMEOUT);
 }
 
-// Reference value of element e (segment-local) whose normal is z.
-__device__ __forceinline__ float ref_value(float z, uint32_t c, const GenParams &p,
-                                           const uint32_t *outlier_mask) {
-  if (p.n_outlier > 0 && mask_bit(outlier_mask, c)) return z * p.outlier_scale;
-  return z;
-}
-
-// ----------------------------------------------------------------- pass 1: references
-// Work item = (segment, chunk of kGenStatChunk elements).  Each thread takes
-// groups of 8 elements: two Philox blocks of reference normals, the
-// reference a (outlier channels scaled), a 16-byte store pair when the
-// group is whole and 8-aligned.  The block also reduces what the live values
-// need: sum |a| on a benign stage under the Eq. 2 model (mu = ||a||_1 / (T d));
-// sum a^2 and the tamper direction's sum g^2 on a Gaussian-tamper stage
-// (tau(v) = v + eps ||v|| g / ||g||).  One double2 per item.
+// The eight normals of elements e0 .. e0 + 7 (blocks q0 = e0 / 4 and q0 + 1
+// of counter (q, seg, c2, c3)); the second block only when the group has
+// more than four elements.
 __device__ __forceinline__ void normals8(const PhiloxRoundKeys &rk, uint32_t q0, uint32_t seg,
                                          uint32_t c2, uint32_t c3, int cnt, float z[8]) {
   const float4 a = normals4_rk(rk, q0, seg, c2, c3);
@@ -115,54 +107,162 @@ __device__ __forceinline__ void normals8(const PhiloxRoundKeys &rk, uint32_t q0,
   }
 }
 
+// Bits 0..7 = mask bits of the channels c, c+1, ..., c+7 (wrapping at d).
+// When 8 divides d, c (= e0 mod d with e0 a multiple of 8) is a multiple of
+// 8, so the eight channels sit in one mask word and one load serves them.
+__device__ __forceinline__ uint32_t channel_bits8(const uint32_t *mask, uint32_t c, uint32_t d) {
+  if ((d & 7u) == 0) return (__ldg(mask + (c >> 5)) >> (c & 31u)) & 0xFFu;
+  uint32_t bits = 0;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    bits |= (mask_bit(mask, c) ? 1u : 0u) << k;
+    c = (c + 1 == d) ? 0 : c + 1;
+  }
+  return bits;
+}
+
+// Whether a stage's live values depend on statistics of the whole segment:
+// benign under the Eq. 2 model (mu = ||a||_1 / (T d)), malicious under the
+// Gaussian tamper (||v||, ||g||).  Every other segment's live values follow
+// element by element from its references.
+__device__ __forceinline__ bool needs_stats(const GenParams &p, bool mal) {
+  return mal ? p.tamper == CG_TAMPER_ADDITIVE : p.noise == CG_NOISE_PAPER;
+}
+
+// fp16 live values of one group of 8, or in recompute mode their fp32
+// copies written over the references.
+__device__ __forceinline__ void store_live(const GenParams &p, uint16_t *acts, float *refs,
+                                           uint64_t g, int cnt, bool vec, const float h[8]) {
+  if (p.recompute) {
+    if (vec) {
+      float v[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) v[k] = __half2float(__float2half_rn(h[k]));
+      float4 *r4 = reinterpret_cast<float4 *>(refs + g);
+      r4[0] = make_float4(v[0], v[1], v[2], v[3]);
+      r4[1] = make_float4(v[4], v[5], v[6], v[7]);
+    } else {
+      for (int k = 0; k < cnt; ++k) refs[g + k] = __half2float(__float2half_rn(h[k]));
+    }
+    return;
+  }
+  if (vec) {
+    uint4 hv;
+    hv.x = (uint32_t)__half_as_ushort(__float2half_rn(h[0])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(h[1])) << 16);
+    hv.y = (uint32_t)__half_as_ushort(__float2half_rn(h[2])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(h[3])) << 16);
+    hv.z = (uint32_t)__half_as_ushort(__float2half_rn(h[4])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(h[5])) << 16);
+    hv.w = (uint32_t)__half_as_ushort(__float2half_rn(h[6])) |
+           ((uint32_t)__half_as_ushort(__float2half_rn(h[7])) << 16);
+    *reinterpret_cast<uint4 *>(acts + g) = hv;
+  } else {
+    for (int k = 0; k < cnt; ++k) acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
+  }
+}
+
+// ----------------------------------------------------------------- pass 1: references
+// Work item = (segment, chunk of kGenStatChunk elements).  Each thread takes
+// groups of 8 elements: two Philox blocks of reference normals, the
+// reference a (outlier channels scaled), a 16-byte store pair when the
+// group is whole and 8-aligned.
+// kLive: on a segment whose live values need no segment statistics (benign
+// a (1 + sigma_s z); sign flips; rescale) the live values are formed here
+// from the registers and stored beside the references, and pass 2 skips
+// the segment.  On the other segments the block reduces what their live
+// values need: sum |a| on a benign stage under the Eq. 2 model, sum a^2 and
+// the tamper direction's sum g^2 on a Gaussian-tamper stage.  One double2
+// per item.  Without kLive only the references are written.
+template <bool kLive>
 __global__ void __launch_bounds__(kGenThreads)
-gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *__restrict__ refs,
+gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask,
+                const uint32_t *__restrict__ flip_mask, const float *__restrict__ stage_sigma,
+                float *__restrict__ refs, uint16_t *__restrict__ acts,
                 double2 *__restrict__ stats) {
   __shared__ double2 warp_sum[kGenThreads / 32];
   const uint64_t n_items = (uint64_t)p.S * p.N * p.stat_chunks;
   const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_ref = 4u * p.config_id + kStreamRef;
+  const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
+  const uint32_t c_step = (uint32_t)((8ull * kGenThreads) % p.d);
   const int tid = threadIdx.x;
   for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x) {
     const uint32_t seg = (uint32_t)(item / p.stat_chunks);
     const uint64_t ch = item - (uint64_t)seg * p.stat_chunks;
     const uint32_t s = seg / p.N;
     const bool mal = is_malicious(p, s);
-    const bool need_l1 = !mal && p.noise == CG_NOISE_PAPER;
-    const bool need_l2 = mal && p.tamper == CG_TAMPER_ADDITIVE;
+    const bool stat_seg = kLive && needs_stats(p, mal);
+    const bool fused = kLive && !stat_seg;
+    const bool need_l1 = stat_seg && !mal;
+    const bool need_l2 = stat_seg && mal;
+    const bool flips = fused && mal && p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS;
+    // the per-segment scalar of a fused segment: sigma_s (benign) or beta (rescale)
+    const float cf = !fused ? 0.f : (mal ? p.tamper_param : stage_sigma[s]);
+    const uint32_t *flip_row = flip_mask + (uint64_t)s * p.mask_words;
+    const uint64_t seg_base = (uint64_t)seg * p.L;
     const uint64_t e_begin = ch * kGenStatChunk;
     const uint64_t e_end = min(e_begin + (uint64_t)kGenStatChunk, p.L);
+    uint64_t e0 = e_begin + 8 * (uint64_t)tid;
+    uint32_t c = (uint32_t)(e0 % p.d);                   // channel of element e0
     float x = 0.f, y = 0.f;
-    for (uint64_t e0 = e_begin + 8 * (uint64_t)tid; e0 < e_end; e0 += 8 * (uint64_t)kGenThreads) {
+    for (; e0 < e_end; e0 += 8 * (uint64_t)kGenThreads) {
       const int cnt = (int)min((uint64_t)8, p.L - e0);
+      const uint32_t q0 = (uint32_t)(e0 >> 2);
       float z[8], a[8];
-      normals8(rk, (uint32_t)(e0 >> 2), seg, c2_ref, 0u, cnt, z);
-      uint32_t c = (uint32_t)(e0 % p.d);
+      normals8(rk, q0, seg, c2_ref, 0u, cnt, z);
+      const uint32_t obits = p.n_outlier > 0 ? channel_bits8(outlier_mask, c, p.d) : 0u;
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        a[k] = ref_value(z[k], c, p, outlier_mask);
-        c = (c + 1 == p.d) ? 0 : c + 1;
-      }
+      for (int k = 0; k < 8; ++k) a[k] = ((obits >> k) & 1u) ? z[k] * p.outlier_scale : z[k];
+      const uint64_t gidx = seg_base + e0;
+      const bool vec = cnt == 8 && (gidx & 7) == 0;
       if (need_l1) {
         for (int k = 0; k < cnt; ++k) x += fabsf(a[k]);
       } else if (need_l2) {
         float g[8];
-        normals8(rk, (uint32_t)(e0 >> 2), seg, c2_tamper, 0u, cnt, g);
+        normals8(rk, q0, seg, c2_tamper, 0u, cnt, g);
         for (int k = 0; k < cnt; ++k) {
           x = fmaf(a[k], a[k], x);
           y = fmaf(g[k], g[k], y);
         }
       }
-      const uint64_t gidx = (uint64_t)seg * p.L + e0;
-      if (cnt == 8 && (gidx & 7) == 0) {
+      if (fused) {
+        float h[8];
+        if (!mal) {
+          float n[8];
+          normals8(rk, q0, seg, c2_noise, p.noise_c3, cnt, n);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) h[k] = a[k] * (1.0f + cf * n[k]);   // a (1 + sigma_s z)
+        } else if (flips) {
+          const uint32_t fbits = channel_bits8(flip_row, c, p.d);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) h[k] = ((fbits >> k) & 1u) ? -a[k] : a[k];
+        } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) h[k] = -a[k];
+        } else {
+#pragma unroll
+          for (int k = 0; k < 8; ++k) h[k] = cf * a[k];                    // beta a
+        }
+        store_live(p, acts, refs, gidx, cnt, vec, h);
+        if (p.recompute) {
+          c += c_step;
+          if (c >= p.d) c -= p.d;
+          continue;                                   // the recompute replaces the references
+        }
+      }
+      if (vec) {
         float4 *r4 = reinterpret_cast<float4 *>(refs + gidx);
         r4[0] = make_float4(a[0], a[1], a[2], a[3]);
         r4[1] = make_float4(a[4], a[5], a[6], a[7]);
       } else {
         for (int k = 0; k < cnt; ++k) refs[gidx + k] = a[k];
       }
+      c += c_step;
+      if (c >= p.d) c -= p.d;
     }
+    if (!stat_seg) continue;                         // uniform over the block
     double dx = x, dy = y;
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
@@ -184,14 +284,19 @@ gen_refs_kernel(GenParams p, const uint32_t *__restrict__ outlier_mask, float *_
 }
 
 // ----------------------------------------------------------------- coef
-// Per segment: benign MULT -> sigma_s; benign PAPER -> sigma_s * mu with
-// mu = sum|a| / L (Eq. 2); malicious ADDITIVE -> eps sqrt(sum a^2 / sum g^2)
-// (tau(v) = v + eps ||v|| g / ||g||); SCALE -> beta; otherwise 0.
-__global__ void gen_coef_kernel(GenParams p, const double2 *__restrict__ stats,
+// Per segment of stages s_first .. s_first + n_stages - 1: benign PAPER ->
+// sigma_s * mu with mu = sum|a| / L (Eq. 2); malicious ADDITIVE ->
+// eps sqrt(sum a^2 / sum g^2) (tau(v) = v + eps ||v|| g / ||g||); benign
+// MULT -> sigma_s; SCALE -> beta; otherwise 0.  stat_only: only the
+// segments whose live values need statistics (the others were finished in
+// pass 1 and have no sums).  Fixed order, fp64.
+__global__ void gen_coef_kernel(GenParams p, uint32_t s_first, uint32_t n_stages, int stat_only,
+                                const double2 *__restrict__ stats,
                                 const float *__restrict__ stage_sigma, float *__restrict__ coef) {
-  const uint64_t seg = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (seg >= (uint64_t)p.S * p.N) return;
+  const uint64_t seg = (uint64_t)s_first * p.N + (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (seg >= (uint64_t)(s_first + n_stages) * p.N) return;
   const uint32_t s = (uint32_t)(seg / p.N);
+  if (stat_only && !needs_stats(p, is_malicious(p, s))) return;
   double x = 0.0, y = 0.0;
   const double2 *st = stats + seg * p.stat_chunks;
   for (uint64_t c = 0; c < p.stat_chunks; ++c) {
@@ -211,97 +316,54 @@ __global__ void gen_coef_kernel(GenParams p, const double2 *__restrict__ stats,
 }
 
 // ----------------------------------------------------------------- pass 2: live values
-// One thread per group of 8 segment-local elements: the references written
-// by pass 1 are read back (16-byte loads when the group is whole and
-// 8-aligned), the benign noise or the tamper applied, the fp16 live values
-// stored.  In recompute mode every stage is benign, its noise comes from
-// counter word 3 = the replica, and the fp16 result overwrites the
-// references in place as fp32.
+// The segments pass 1 left: benign under the Eq. 2 model (h = a + sigma_s mu
+// z) and malicious under the Gaussian tamper (h = a + coef g), both
+// h = fp16(a + coef w) with w the noise or tamper normal.  Work item =
+// (segment, chunk of kLiveChunk elements); each thread takes groups of 8:
+// the references read back (16-byte loads when the group is whole and
+// 8-aligned), the normals drawn, the fp16 live values stored.  In recompute
+// mode every stage is benign, its noise comes from counter word 3 = the
+// replica, and the fp16 result overwrites the references in place as fp32.
+constexpr uint64_t kLiveChunk = 8 * kGenThreads * 8;
+
 __global__ void __launch_bounds__(kGenThreads)
-gen_live_kernel(GenParams p, const uint32_t *__restrict__ flip_mask, const float *__restrict__ coef,
-                uint16_t *__restrict__ acts, float *__restrict__ refs) {
-  const uint64_t groups_per_seg = (p.L + 7) >> 3;
-  const uint64_t total = (uint64_t)p.S * p.N * groups_per_seg;
+gen_live_kernel(GenParams p, const float *__restrict__ coef, uint16_t *__restrict__ acts,
+                float *__restrict__ refs) {
+  const uint64_t chunks = (p.L + kLiveChunk - 1) / kLiveChunk;
+  const uint64_t n_items = (uint64_t)p.S * p.N * chunks;
   const PhiloxRoundKeys &rk = *reinterpret_cast<const PhiloxRoundKeys *>(p.round_keys);
   const uint32_t c2_noise = 4u * p.config_id + kStreamNoise;
   const uint32_t c2_tamper = 4u * p.config_id + kStreamTamper;
-  for (uint64_t gi = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; gi < total;
-       gi += (uint64_t)gridDim.x * blockDim.x) {
-    const uint32_t seg = (uint32_t)(gi / groups_per_seg);
-    const uint64_t j = gi - (uint64_t)seg * groups_per_seg;
+  for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x) {
+    const uint32_t seg = (uint32_t)(item / chunks);
     const uint32_t s = seg / p.N;
-    const uint64_t e0 = 8 * j;
-    const int cnt = (int)min((uint64_t)8, p.L - e0);
-    const uint32_t q0 = (uint32_t)(2 * j);
-    const uint64_t g = (uint64_t)seg * p.L + e0;
-    const bool vec = (cnt == 8) && ((g & 7) == 0);
-
-    float a[8], h[8];
-    if (vec) {
-      const float4 r0 = reinterpret_cast<const float4 *>(refs + g)[0];
-      const float4 r1 = reinterpret_cast<const float4 *>(refs + g)[1];
-      a[0] = r0.x; a[1] = r0.y; a[2] = r0.z; a[3] = r0.w;
-      a[4] = r1.x; a[5] = r1.y; a[6] = r1.z; a[7] = r1.w;
-    } else {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) a[k] = (k < cnt) ? refs[g + k] : 0.f;
-    }
-
     const bool mal = is_malicious(p, s);
+    if (!needs_stats(p, mal)) continue;
+    const uint64_t ch = item - (uint64_t)seg * chunks;
     const float cf = coef[seg];
-    if (!mal || p.tamper == CG_TAMPER_ADDITIVE) {
-      float n[8];
-      normals8(rk, q0, seg, mal ? c2_tamper : c2_noise, mal ? 0u : p.noise_c3, cnt, n);
-      if (!mal && p.noise == CG_NOISE_MULT) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) h[k] = a[k] * (1.0f + cf * n[k]);   // a (1 + sigma_s z)
-      } else {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) h[k] = fmaf(cf, n[k], a[k]);        // a + coef z
-      }
-    } else if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS) {
-      const uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
-      uint32_t c = (uint32_t)(e0 % p.d);
-#pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        h[k] = mask_bit(row, c) ? -a[k] : a[k];
-        c = (c + 1 == p.d) ? 0 : c + 1;
-      }
-    } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) h[k] = -a[k];
-    } else {
-#pragma unroll
-      for (int k = 0; k < 8; ++k) h[k] = cf * a[k];
-    }
-
-    if (p.recompute) {
-      // independent benign recompute: the fp16 output, stored as fp32 in place
+    const uint32_t c2 = mal ? c2_tamper : c2_noise;
+    const uint32_t c3 = mal ? 0u : p.noise_c3;
+    const uint64_t seg_base = (uint64_t)seg * p.L;
+    const uint64_t e_end = min((ch + 1) * kLiveChunk, p.L);
+    for (uint64_t e0 = ch * kLiveChunk + 8 * (uint64_t)threadIdx.x; e0 < e_end;
+         e0 += 8 * (uint64_t)kGenThreads) {
+      const int cnt = (int)min((uint64_t)8, p.L - e0);
+      const uint64_t g = seg_base + e0;
+      const bool vec = cnt == 8 && (g & 7) == 0;
+      float a[8], w[8], h[8];
       if (vec) {
-        float v[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) v[k] = __half2float(__float2half_rn(h[k]));
-        float4 *r4 = reinterpret_cast<float4 *>(refs + g);
-        r4[0] = make_float4(v[0], v[1], v[2], v[3]);
-        r4[1] = make_float4(v[4], v[5], v[6], v[7]);
+        const float4 r0 = reinterpret_cast<const float4 *>(refs + g)[0];
+        const float4 r1 = reinterpret_cast<const float4 *>(refs + g)[1];
+        a[0] = r0.x; a[1] = r0.y; a[2] = r0.z; a[3] = r0.w;
+        a[4] = r1.x; a[5] = r1.y; a[6] = r1.z; a[7] = r1.w;
       } else {
-        for (int k = 0; k < cnt; ++k) refs[g + k] = __half2float(__float2half_rn(h[k]));
+#pragma unroll
+        for (int k = 0; k < 8; ++k) a[k] = (k < cnt) ? refs[g + k] : 0.f;
       }
-      continue;
-    }
-    if (vec) {
-      uint4 hv;
-      hv.x = (uint32_t)__half_as_ushort(__float2half_rn(h[0])) |
-             ((uint32_t)__half_as_ushort(__float2half_rn(h[1])) << 16);
-      hv.y = (uint32_t)__half_as_ushort(__float2half_rn(h[2])) |
-             ((uint32_t)__half_as_ushort(__float2half_rn(h[3])) << 16);
-      hv.z = (uint32_t)__half_as_ushort(__float2half_rn(h[4])) |
-             ((uint32_t)__half_as_ushort(__float2half_rn(h[5])) << 16);
-      hv.w = (uint32_t)__half_as_ushort(__float2half_rn(h[6])) |
-             ((uint32_t)__half_as_ushort(__float2half_rn(h[7])) << 16);
-      *reinterpret_cast<uint4 *>(acts + g) = hv;
-    } else {
-      for (int k = 0; k < cnt; ++k) acts[g + k] = __half_as_ushort(__float2half_rn(h[k]));
+      normals8(rk, (uint32_t)(e0 >> 2), seg, c2, c3, cnt, w);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) h[k] = fmaf(cf, w[k], a[k]);           // a + coef w
+      store_live(p, acts, refs, g, cnt, vec, h);
     }
   }
 }
@@ -448,13 +510,10 @@ gen_prop_live_kernel(GenParams p, uint32_t s, float gain, const uint32_t *__rest
         for (int k = 0; k < 8; ++k) h[k] = fmaf(cf, z[k], v[k]);
       }
     } else if (p.tamper == CG_TAMPER_SIGNFLIP_CHANNELS) {
-      const uint32_t *row = flip_mask + (uint64_t)s * p.mask_words;
-      uint32_t c = (uint32_t)(e0 % p.d);
+      const uint32_t fbits =
+          channel_bits8(flip_mask + (uint64_t)s * p.mask_words, (uint32_t)(e0 % p.d), p.d);
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        h[k] = mask_bit(row, c) ? -v[k] : v[k];
-        c = (c + 1 == p.d) ? 0 : c + 1;
-      }
+      for (int k = 0; k < 8; ++k) h[k] = ((fbits >> k) & 1u) ? -v[k] : v[k];
     } else if (p.tamper == CG_TAMPER_SIGNFLIP_FULL) {
 #pragma unroll
       for (int k = 0; k < 8; ++k) h[k] = -v[k];
@@ -510,6 +569,16 @@ __global__ void philox_normals_kernel(uint64_t seed, uint32_t c1, uint32_t c2, u
   out[i] = make_float4(a.x, a.y, b.x, b.y);
 }
 
+// Whether any segment's live values need segment statistics (pass 2).
+bool host_any_stats(const GenParams &p) {
+  bool any_mal = false, any_benign = false;
+  for (uint32_t s = 0; s < p.S; ++s) {
+    if ((p.mal_bits[s >> 5] >> (s & 31)) & 1u) any_mal = true;
+    else any_benign = true;
+  }
+  return (any_benign && p.noise == CG_NOISE_PAPER) || (any_mal && p.tamper == CG_TAMPER_ADDITIVE);
+}
+
 }  // namespace
 
 GenLayout gen_layout(const cg_pipeline_desc &d) {
@@ -552,15 +621,17 @@ cudaError_t launch_generate(const GenParams &p, uint16_t *acts, float *refs, int
   const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)info.gen_blocks_per_sm;
   const uint64_t n_items = n_seg * p.stat_chunks;
   const uint64_t grid1 = n_items < resident ? n_items : resident;
-  gen_refs_kernel<<<(unsigned)grid1, kGenThreads, 0, stream>>>(p, outlier_mask, refs, stats);
+  gen_refs_kernel<true><<<(unsigned)grid1, kGenThreads, 0, stream>>>(
+      p, outlier_mask, flip_mask, stage_sigma, refs, acts, stats);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
-  gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, stats, stage_sigma, coef);
-  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  if (!host_any_stats(p)) return cudaSuccess;       // pass 1 finished every segment
 
-  const uint64_t groups = n_seg * ((p.L + 7) >> 3);
-  const uint64_t blocks_needed = (groups + kGenThreads - 1) / kGenThreads;
-  const uint64_t grid = blocks_needed < resident * 4 ? blocks_needed : resident * 4;
-  gen_live_kernel<<<(unsigned)grid, kGenThreads, 0, stream>>>(p, flip_mask, coef, acts, refs);
+  gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, 0, p.S, 1, stats,
+                                                                       stage_sigma, coef);
+  if ((err = cudaGetLastError()) != cudaSuccess) return err;
+  const uint64_t live_items = n_seg * ((p.L + kLiveChunk - 1) / kLiveChunk);
+  const uint64_t grid2 = live_items < resident ? live_items : resident;
+  gen_live_kernel<<<(unsigned)grid2, kGenThreads, 0, stream>>>(p, coef, acts, refs);
   return cudaGetLastError();
 }
 
@@ -582,8 +653,8 @@ cudaError_t launch_generate_propagating(const GenParams &p, float gain, uint16_t
   const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)info.gen_blocks_per_sm;
   // every stage's reference first (its statistics are recomputed below)
   const uint64_t n_items = n_seg * p.stat_chunks;
-  gen_refs_kernel<<<(unsigned)(n_items < resident ? n_items : resident), kGenThreads, 0, stream>>>(
-      p, outlier_mask, refs, stats);
+  gen_refs_kernel<false><<<(unsigned)(n_items < resident ? n_items : resident), kGenThreads, 0,
+                          stream>>>(p, outlier_mask, flip_mask, stage_sigma, refs, nullptr, nullptr);
   if ((err = cudaGetLastError()) != cudaSuccess) return err;
   const uint64_t stage_items = (uint64_t)p.N * p.stat_chunks;
   const uint64_t stage_groups = (uint64_t)p.N * ((p.L + 7) >> 3);
@@ -592,8 +663,8 @@ cudaError_t launch_generate_propagating(const GenParams &p, float gain, uint16_t
     gen_prop_stats_kernel<<<(unsigned)(stage_items < resident ? stage_items : resident), kGenThreads,
                             0, stream>>>(p, s, gain, refs, acts, stats);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
-    gen_coef_kernel<<<(unsigned)((n_seg + 127) / 128), 128, 0, stream>>>(p, stats, stage_sigma,
-                                                                         coef);
+    gen_coef_kernel<<<(unsigned)((p.N + 127) / 128), 128, 0, stream>>>(p, s, 1, 0, stats,
+                                                                       stage_sigma, coef);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     gen_prop_live_kernel<<<(unsigned)(live_blocks < resident * 4 ? live_blocks : resident * 4),
                            kGenThreads, 0, stream>>>(p, s, gain, flip_mask, coef, refs, acts);
@@ -626,7 +697,7 @@ cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint3
 
 int gen_occupancy() {
   int n = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_live_kernel, kGenThreads, 0) !=
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_refs_kernel<true>, kGenThreads, 0) !=
       cudaSuccess)
     return 0;
   return n;
