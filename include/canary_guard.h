@@ -130,6 +130,18 @@ cg_status cg_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3
                             uint32_t first_block, uint32_t n_blocks,
                             float *d_out, cg_stream_t stream);
 
+/*
+ * The Box-Muller transform alone, on caller-given word pairs: pair i =
+ * (d_words[2i], d_words[2i+1]) -> d_out[2i], d_out[2i+1] = sqrt(-2 ln u1)
+ * (cos, sin)(2 pi u2) with u1 = ((x0 >> 8) + 1) 2^-24 and u2 = (x1 >> 8)
+ * 2^-24, in fp32, by the same device code every generator normal goes
+ * through.  It lets a test sweep each factor over all 2^24 values of its
+ * word.  d_words: 2 * n_pairs words, d_out: 2 * n_pairs floats, both device
+ * memory, 8-byte aligned.  n_pairs = 0 or a null pointer -> INVALID_ARG.
+ */
+cg_status cg_box_muller_pairs(const uint32_t *d_words, uint64_t n_pairs, float *d_out,
+                              cg_stream_t stream);
+
 /* Workspace bytes cg_generate_pipeline needs for `desc`. */
 cg_status cg_generate_workspace_size(const cg_pipeline_desc *desc, size_t *bytes);
 

@@ -114,6 +114,12 @@ void or_box_muller(uint32_t x0, uint32_t x1, double *z0, double *z1) {
   *z1 = r * sin(theta);
 }
 
+/* The transform over word pairs: pair i = (words[2i], words[2i+1]). */
+void or_box_muller_pairs(const uint32_t *words, uint64_t n_pairs, double *out) {
+  for (uint64_t i = 0; i < n_pairs; ++i)
+    or_box_muller(words[2 * i], words[2 * i + 1], out + 2 * i, out + 2 * i + 1);
+}
+
 /* Normals of blocks [first_block, first_block + n_blocks): 4 per block,     */
 /* (x0, x1) -> elements 0, 1 and (x2, x3) -> elements 2, 3.                  */
 void or_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,

@@ -80,6 +80,7 @@ def lib():
             L.or_philox4x32_10.argtypes = [P(u32), P(u32), P(u32)]
             L.or_philox_words.argtypes = [u64, u32, u32, u32, u32, u32, P(u32)]
             L.or_box_muller.argtypes = [u32, u32, P(dbl), P(dbl)]
+            L.or_box_muller_pairs.argtypes = [P(u32), u64, P(dbl)]
             L.or_philox_normals.argtypes = [u64, u32, u32, u32, u32, u32, P(dbl)]
             L.or_aux_bounded.argtypes = [u64, u32, u32, u32, u32, u32, P(u32)]
             L.or_half_from_double.argtypes = [dbl]
@@ -152,6 +153,14 @@ def box_muller(x0, x1):
     z0, z1 = ctypes.c_double(), ctypes.c_double()
     lib().or_box_muller(int(x0), int(x1), ctypes.byref(z0), ctypes.byref(z1))
     return z0.value, z1.value
+
+
+def box_muller_pairs(words):
+    """Box-Muller of word pairs: words uint32 [n, 2] -> float64 [n, 2]."""
+    w = np.ascontiguousarray(words, dtype=np.uint32).reshape(-1, 2)
+    out = np.zeros(w.shape, dtype=np.float64)
+    lib().or_box_muller_pairs(_p(w, ctypes.c_uint32), w.shape[0], _p(out, ctypes.c_double))
+    return out
 
 
 def philox_normals(seed, c1, c2, c3, first_block, n_blocks):

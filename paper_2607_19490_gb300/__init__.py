@@ -18,7 +18,7 @@ from .build import LIB_PATH, build  # noqa: F401
 
 __all__ = [
     "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
-    "cg_philox_words", "cg_philox_normals", "cg_generate_workspace_size",
+    "cg_philox_words", "cg_philox_normals", "cg_box_muller_pairs", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
     "cg_drift_scores_ex", "cg_drift_scores_host", "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
@@ -93,6 +93,7 @@ def load() -> ctypes.CDLL:
             "cg_abi_version": ([], ctypes.c_int),
             "cg_philox_words": ([u64, u32, u32, u32, u32, u32, P, P], ctypes.c_int),
             "cg_philox_normals": ([u64, u32, u32, u32, u32, u32, P, P], ctypes.c_int),
+            "cg_box_muller_pairs": ([P, u64, P, P], ctypes.c_int),
             "cg_generate_workspace_size": ([ctypes.POINTER(PipelineDesc), ctypes.POINTER(sz)], ctypes.c_int),
             "cg_generate_pipeline": ([ctypes.POINTER(PipelineDesc), P, P, P, P, sz, P, P], ctypes.c_int),
             "cg_drift_workspace_size": ([u32, u32, u64, ctypes.POINTER(sz)], ctypes.c_int),
@@ -182,6 +183,24 @@ def cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, out=None, stream=
         raise ValueError("out must hold 4 * n_blocks floats")
     _check(load().cg_philox_normals(seed, c1, c2, c3, first_block, n_blocks, _ptr(out),
                                     _stream(stream)), "cg_philox_normals")
+    return out
+
+
+def cg_box_muller_pairs(words, out=None, stream=None):
+    """Box-Muller of word pairs: words int32 [n, 2] (uint32 bit patterns) on
+    the device -> float32 [n, 2] = (z0, z1) per pair."""
+    torch = _torch()
+    _cuda(words, "words", (torch.int32,))
+    if words.numel() % 2 or words.numel() == 0:
+        raise ValueError("words must hold a positive even number of words")
+    n = words.numel() // 2
+    if out is None:
+        out = torch.empty((n, 2), dtype=torch.float32, device="cuda")
+    _cuda(out, "out", (torch.float32,))
+    if out.numel() < 2 * n:
+        raise ValueError("out must hold 2 * n floats")
+    _check(load().cg_box_muller_pairs(_ptr(words), n, _ptr(out), _stream(stream)),
+           "cg_box_muller_pairs")
     return out
 
 

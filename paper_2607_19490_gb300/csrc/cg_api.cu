@@ -179,6 +179,14 @@ cg_status cg_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3
                                              (cudaStream_t)stream));
 }
 
+cg_status cg_box_muller_pairs(const uint32_t *d_words, uint64_t n_pairs, float *d_out,
+                              cg_stream_t stream) {
+  CG_TRACE("cg_box_muller_pairs");
+  if (!d_words || !d_out || n_pairs == 0) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_words, 8) || !aligned(d_out, 8)) return CG_ERR_ALIGNMENT;
+  return from_cuda(cg::launch_box_muller_pairs(d_words, n_pairs, d_out, (cudaStream_t)stream));
+}
+
 cg_status cg_generate_workspace_size(const cg_pipeline_desc *desc, size_t *bytes) {
   if (!bytes) return CG_ERR_INVALID_ARG;
   cg_status st = check_desc(desc);

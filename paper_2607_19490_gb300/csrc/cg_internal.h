@@ -88,6 +88,8 @@ cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C,
 
 cudaError_t launch_philox_words(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
                                 uint32_t first, uint32_t n, uint32_t *out, cudaStream_t stream);
+cudaError_t launch_box_muller_pairs(const uint32_t *words, uint64_t n_pairs, float *out,
+                                   cudaStream_t stream);
 cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint32_t c3,
                                   uint32_t first, uint32_t n, float *out, cudaStream_t stream);
 

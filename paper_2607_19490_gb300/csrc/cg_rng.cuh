@@ -59,16 +59,55 @@ __device__ __forceinline__ uint2 philox_key(uint64_t seed) {
   return make_uint2((uint32_t)seed, (uint32_t)(seed >> 32));
 }
 
+// (sin, cos)(2 pi k 2^-24) for a 24-bit k.  The angle is pi t with
+// t = k 2^-23, so the reduction to the nearest quarter turn q and the
+// remainder r = t - q / 2 in [-1/4, 1/4] is integer arithmetic and exact.
+// On the remainder, sin(pi r) and cos(pi r) are their Taylor series about 0
+// through r^9 and r^10 (coefficients (-1)^j pi^(2j+1) / (2j+1)! and
+// (-1)^j pi^(2j) / (2j)!); the first omitted terms are below 3e-9 and
+// 1.2e-10 of the result at |r| = 1/4.  The quadrant then swaps the pair and
+// sets the signs.  Over all 2^24 arguments the result is within 3.4 units
+// of 2^-24 relative of the exact value.
+__device__ __forceinline__ float2 sincos_2pi_u24(uint32_t k) {
+  const uint32_t q = (k + (1u << 21)) >> 22;           // round(2 t), 0 .. 4
+  const float r = (float)((int32_t)k - (int32_t)(q << 22)) * 0x1p-23f;
+  const float r2 = r * r;
+  float ps = 0.08214588661112819f;                     //  pi^9 / 9!
+  ps = fmaf(ps, r2, -0.5992645293207919f);             // -pi^7 / 7!
+  ps = fmaf(ps, r2, 2.550164039877345f);               //  pi^5 / 5!
+  ps = fmaf(ps, r2, -5.167712780049969f);              // -pi^3 / 3!
+  ps = fmaf(ps, r2, 3.141592653589793f);               //  pi
+  const float sr = ps * r;                             // sin(pi r)
+  float pc = -0.02580689139001405f;                    // -pi^10 / 10!
+  pc = fmaf(pc, r2, 0.23533063035889312f);             //  pi^8 / 8!
+  pc = fmaf(pc, r2, -1.3352627688545893f);             // -pi^6 / 6!
+  pc = fmaf(pc, r2, 4.058712126416768f);               //  pi^4 / 4!
+  pc = fmaf(pc, r2, -4.934802200544679f);              // -pi^2 / 2!
+  const float cr = fmaf(pc, r2, 1.0f);                 // cos(pi r)
+  const bool odd = q & 1u;                             // a quarter turn swaps sin and cos
+  const uint32_t s_neg = (q & 2u) << 30;               // q = 2, 3: sin < 0
+  const uint32_t c_neg = ((q + 1u) & 2u) << 30;        // q = 1, 2: cos < 0
+  return make_float2(__uint_as_float(__float_as_uint(odd ? sr : cr) ^ c_neg),
+                     __uint_as_float(__float_as_uint(odd ? cr : sr) ^ s_neg));   // (cos, sin)
+}
+
+// PTX's approximate square root (one special-function instruction).  Over
+// every argument -2 ln u1 takes here it is within 2.3 units of 2^-24
+// relative of the exact root, and exactly 0 at 0.
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float y;
+  asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Box-Muller on two words: u1 = ((x0 >> 8) + 1) 2^-24 in (0, 1],
 // u2 = (x1 >> 8) 2^-24 in [0, 1); (z0, z1) = sqrt(-2 ln u1) (cos, sin)(2 pi u2).
-// Both uniforms are exact in fp32; sincospif takes the exact 2 u2.
+// u1 is exact in fp32; the angle is taken from the integer x1 >> 8.
 __device__ __forceinline__ float2 box_muller(uint32_t x0, uint32_t x1) {
   const float u1 = (float)((x0 >> 8) + 1u) * 0x1p-24f;
-  const float u2 = (float)(x1 >> 8) * 0x1p-24f;
-  const float r = sqrtf(-2.0f * logf(u1));
-  float s, c;
-  sincospif(2.0f * u2, &s, &c);
-  return make_float2(r * c, r * s);
+  const float r = sqrt_approx(-2.0f * logf(u1));
+  const float2 cs = sincos_2pi_u24(x1 >> 8);
+  return make_float2(r * cs.x, r * cs.y);
 }
 
 // The four normals of one Philox block from precomputed round keys.

@@ -569,6 +569,15 @@ __global__ void philox_normals_kernel(uint64_t seed, uint32_t c1, uint32_t c2, u
   out[i] = make_float4(a.x, a.y, b.x, b.y);
 }
 
+__global__ void box_muller_pairs_kernel(const uint2 *__restrict__ words, uint64_t n,
+                                        float2 *__restrict__ out) {
+  for (uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n;
+       i += (uint64_t)gridDim.x * blockDim.x) {
+    const uint2 w = words[i];
+    out[i] = box_muller(w.x, w.y);
+  }
+}
+
 // Whether any segment's live values need segment statistics (pass 2).
 bool host_any_stats(const GenParams &p) {
   bool any_mal = false, any_benign = false;
@@ -692,6 +701,14 @@ cudaError_t launch_philox_normals(uint64_t seed, uint32_t c1, uint32_t c2, uint3
                                   uint32_t first, uint32_t n, float *out, cudaStream_t stream) {
   philox_normals_kernel<<<(n + 255) / 256, 256, 0, stream>>>(seed, c1, c2, c3, first, n,
                                                              reinterpret_cast<float4 *>(out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_box_muller_pairs(const uint32_t *words, uint64_t n_pairs, float *out,
+                                   cudaStream_t stream) {
+  const uint64_t blocks = (n_pairs + 255) / 256;
+  box_muller_pairs_kernel<<<(unsigned)(blocks < 65536 ? blocks : 65536), 256, 0, stream>>>(
+      reinterpret_cast<const uint2 *>(words), n_pairs, reinterpret_cast<float2 *>(out));
   return cudaGetLastError();
 }
 

@@ -42,6 +42,30 @@ def test_philox_normals(cg, orc):
         assert_normals_close(g, o)
 
 
+def test_box_muller_exhaustive(cg, orc):
+    """Each factor of the transform over every value of its 24-bit word
+    index: the radius over all x0 >> 8 at angle 0, then the angle over all
+    x1 >> 8 at the largest radius, a radius near 1 and radius 0.  The low 8
+    bits of each word are set to show they are ignored."""
+    import torch
+    k = np.arange(1 << 24, dtype=np.uint32) << 8
+    sweeps = [(k | 0xAB, np.zeros_like(k))]
+    for k1 in (0, int(round(np.exp(-0.5) * 2**24)) - 1, 2**24 - 1):
+        sweeps.append((np.full_like(k, (k1 << 8) | 0x5C), k | 0x3F))
+    for i, (x0, x1) in enumerate(sweeps):
+        w = np.stack([x0, x1], axis=1)
+        g = cg.cg_box_muller_pairs(torch.from_numpy(w.view(np.int32)).cuda()).cpu().numpy()
+        o = orc.box_muller_pairs(w)
+        assert_normals_close(g, o, what=f"sweep {i}")
+        if i == 0:
+            # the radius alone: within 2.5 units of 2^-24 relative; exact 0 at u1 = 1
+            r_g, r_o = g[:, 0].astype(np.float64), o[:, 0]
+            assert np.all(g[:, 1] == 0.0)
+            assert r_g[-1] == 0.0 and r_o[-1] == 0.0
+            assert np.max(np.abs(r_g[:-1] - r_o[:-1]) / r_o[:-1]) <= 2.5 * 2.0**-24
+        del g, o, w
+
+
 CASES = {
     "tiny": SI.TINY,
     "7b_small": SI.shrink(SI.SEVEN_B, n_canaries=4, tokens=4, hidden=512),

@@ -115,6 +115,17 @@ def test_box_muller_special_cases(orc):
     assert z0 == pytest.approx(math.sqrt(48 * math.log(2)), rel=1e-15)
 
 
+def test_box_muller_pairs_is_the_pairwise_transform(orc):
+    """The array form used by the exhaustive device sweep is the scalar
+    transform applied pair by pair."""
+    rng = np.random.default_rng(5)
+    w = rng.integers(0, 2**32, size=(257, 2), dtype=np.uint64).astype(np.uint32)
+    w[0] = (0xFFFFFFFF, 0)
+    z = orc.box_muller_pairs(w)
+    for i in range(w.shape[0]):
+        assert tuple(z[i]) == orc.box_muller(int(w[i, 0]), int(w[i, 1]))
+
+
 def test_normals_distribution(orc):
     stats = pytest.importorskip("scipy.stats")
     z = orc.philox_normals(2024, 3, 4, 0, 0, 1 << 16)
