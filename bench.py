@@ -283,7 +283,25 @@ def oracle_baseline(cfg, n_threads, seconds):
     return {"value": elems * passes / el, "unit": "elements/s", "cores": n_threads,
             "kind": "oracle", "sample": oracle_describe(sample, passes, el),
             "single_core": {"value": one["S"] * one["L"] / el1, "unit": "elements/s",
-                            "sample": oracle_describe(one, 1, el1)}}
+                            "sample": oracle_describe(one, 1, el1)},
+            "auroc": oracle_auroc_baseline()}
+
+
+def oracle_auroc_baseline(C=65536, N=64, S=16):
+    """The oracle's brute-force Mann-Whitney counts and A-hat (single-threaded
+    C) on the AUROC stress batch's shape: C configurations x N canaries x S
+    stages of uniform scores, stage 0 malicious, drawn on the host."""
+    from oracle import oracle as O
+    rng = np.random.Generator(np.random.PCG64(7))
+    scores = rng.random((C, N, S), dtype=np.float32)
+    labels = np.zeros((C, N, S), dtype=np.int8)
+    labels[:, :, 0] = 1
+    t0 = time.perf_counter()
+    O.auroc(scores, labels)
+    el = time.perf_counter() - t0
+    return {"value": C / el, "unit": "configs/s", "cores": 1, "kind": "oracle",
+            "sample": f"the stress batch's shape: {C} configurations x {N} canaries x {S} stages, "
+                      f"one pass in {el:.2f} s"}
 
 
 def run_reference(args, ranks: Ranks):
