@@ -182,68 +182,121 @@ auroc_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels
 
 // Lane-per-canary ranking for S <= 32 (SP = S rounded up to 4, 8, 16 or
 // 32): each lane loads its canary's scores and labels into registers
-// (16-byte loads when the rows are 16-byte aligned) and counts, for every
-// malicious stage, the benign stages below it and equal to it.  A warp
-// ranks 32 canaries at once with no cross-lane traffic.
+// (16-byte score loads and SP-byte label loads when the rows are exactly SP
+// wide and aligned) and counts, for every malicious stage, the benign
+// stages below it and equal to it.  A warp ranks 32 canaries at once with
+// no cross-lane traffic.  Labels stay packed four to a word; the stage
+// masks come from exact per-byte zero tests on the words.
 template <int SP>
-__device__ __forceinline__ void lane_counts(const float *__restrict__ scores,
-                                            const int8_t *__restrict__ labels, uint64_t o,
-                                            uint32_t S, bool vec, long long &g, long long &e,
-                                            int &nm, int &nb, bool &saw_nan) {
+struct LaneRow {
   float m[SP];
-  int l[SP];
+  uint32_t lw[SP / 4];      // label bytes; 0xFF (excluded) beyond S
+};
+
+template <int SP>
+__device__ __forceinline__ void lane_load(const float *__restrict__ scores,
+                                          const int8_t *__restrict__ labels, uint64_t o,
+                                          uint32_t S, bool vec, LaneRow<SP> &r) {
   const float *ms = scores + o * S;
   const int8_t *ls = labels + o * S;
   if (vec) {
 #pragma unroll
     for (int k = 0; k < SP; k += 4) {
       const float4 v = *reinterpret_cast<const float4 *>(ms + k);
-      m[k] = v.x; m[k + 1] = v.y; m[k + 2] = v.z; m[k + 3] = v.w;
-      const uint32_t w = *reinterpret_cast<const uint32_t *>(ls + k);
-      l[k] = (int)(int8_t)(w & 0xFFu);
-      l[k + 1] = (int)(int8_t)((w >> 8) & 0xFFu);
-      l[k + 2] = (int)(int8_t)((w >> 16) & 0xFFu);
-      l[k + 3] = (int)(int8_t)(w >> 24);
+      r.m[k] = v.x; r.m[k + 1] = v.y; r.m[k + 2] = v.z; r.m[k + 3] = v.w;
+    }
+    if (SP == 4) {
+      r.lw[0] = *reinterpret_cast<const uint32_t *>(ls);
+    } else if (SP == 8) {
+      const uint2 w = *reinterpret_cast<const uint2 *>(ls);
+      r.lw[0] = w.x; r.lw[1 % (SP / 4)] = w.y;
+    } else {
+#pragma unroll
+      for (int q = 0; q < SP / 16; ++q) {
+        const uint4 w = reinterpret_cast<const uint4 *>(ls)[q];
+        r.lw[(4 * q) % (SP / 4)] = w.x; r.lw[(4 * q + 1) % (SP / 4)] = w.y;
+        r.lw[(4 * q + 2) % (SP / 4)] = w.z; r.lw[(4 * q + 3) % (SP / 4)] = w.w;
+      }
     }
   } else {
 #pragma unroll
+    for (int w = 0; w < SP / 4; ++w) r.lw[w] = 0xFFFFFFFFu;
+#pragma unroll
     for (int k = 0; k < SP; ++k) {
-      m[k] = (uint32_t)k < S ? ms[k] : 0.f;
-      l[k] = (uint32_t)k < S ? (int)ls[k] : -1;
+      const bool in = (uint32_t)k < S;
+      r.m[k] = in ? ms[k] : 0.f;
+      if (in) {
+        const uint32_t sh = 8u * (k & 3);
+        r.lw[k >> 2] = (r.lw[k >> 2] & ~(0xFFu << sh)) | ((uint32_t)(uint8_t)ls[k] << sh);
+      }
     }
   }
-  // stage bitmasks; only the malicious stages are walked, the benign
-  // comparison is unrolled (m_i picked by selects, no dynamic indexing)
-  uint32_t mal = 0u, ben = 0u;
+}
+
+// Stage masks keep stage k at bit 8 (k mod 4) + k / 4: label word w holds
+// stages 4w .. 4w + 3 in its bytes, so its per-byte flags (bits 7, 15, 23,
+// 31) land there with one right shift by 7 - w.  Every mask of a lane uses
+// this order; only popcounts and ANDs combine them.
+__host__ __device__ constexpr int stage_bit(int k) { return 8 * (k & 3) + (k >> 2); }
+
+// Bit 8b + 7 of the result = (byte b of x == 0).  Per byte, the low seven
+// bits plus 0x7F carry into bit 7 exactly when they are not all zero (no
+// carry leaves the byte); OR-ing x adds the byte's own bit 7.
+__device__ __forceinline__ uint32_t zero_byte_flags(uint32_t x) {
+  return ~(((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;
+}
+
+template <int SP>
+__device__ __forceinline__ void lane_rank(const LaneRow<SP> &r, int &g, int &e, int &nm, int &nb,
+                                          bool &saw_nan) {
+  uint32_t mal = 0u, ben = 0u, nan = 0u;
 #pragma unroll
-  for (int k = 0; k < SP; ++k) {
-    if ((l[k] == 0 || l[k] == 1) && is_nan_f(m[k])) saw_nan = true;
-    mal |= (uint32_t)(l[k] == 1) << k;
-    ben |= (uint32_t)(l[k] == 0) << k;
+  for (int w = 0; w < SP / 4; ++w) {
+    ben |= zero_byte_flags(r.lw[w]) >> (7 - w);                 // label 0
+    mal |= zero_byte_flags(r.lw[w] ^ 0x01010101u) >> (7 - w);   // label 1
   }
-  const int cm = __popc(mal), cb = __popc(ben);
+#pragma unroll
+  for (int k = 0; k < SP; ++k) nan |= (uint32_t)is_nan_f(r.m[k]) << stage_bit(k);
+  if (nan & (mal | ben)) saw_nan = true;
+  nm = __popc(mal);
+  nb = __popc(ben);
   int lg = 0, le = 0;
+  // only the malicious stages are walked; m_i is picked by selects (no
+  // dynamic register indexing) and compared with every stage at once
   while (mal) {
     const int i = __ffs(mal) - 1;
     mal &= mal - 1u;
     float mi = 0.f;
 #pragma unroll
-    for (int k = 0; k < SP; ++k) mi = (k == i) ? m[k] : mi;
+    for (int k = 0; k < SP; ++k) mi = (stage_bit(k) == i) ? r.m[k] : mi;
+    uint32_t gtm = 0u, eqm = 0u;
 #pragma unroll
     for (int j = 0; j < SP; ++j) {
-      const bool b = (ben >> j) & 1u;
-      lg += (b && mi > m[j]);
-      le += (b && mi == m[j]);
+      gtm |= (uint32_t)(mi > r.m[j]) << stage_bit(j);
+      eqm |= (uint32_t)(mi == r.m[j]) << stage_bit(j);
     }
+    lg += __popc(gtm & ben);
+    le += __popc(eqm & ben);
   }
   g = lg;
   e = le;
-  nm = cm;
-  nb = cb;
 }
 
 template <int SP>
-__global__ void __launch_bounds__(kRankThreads)
+__device__ __forceinline__ void lane_counts(const float *__restrict__ scores,
+                                            const int8_t *__restrict__ labels, uint64_t o,
+                                            uint32_t S, bool vec, long long &g, long long &e,
+                                            int &nm, int &nb, bool &saw_nan) {
+  LaneRow<SP> r;
+  lane_load<SP>(scores, labels, o, S, vec, r);
+  int gi, ei;
+  lane_rank<SP>(r, gi, ei, nm, nb, saw_nan);
+  g = gi;
+  e = ei;
+}
+
+template <int SP>
+__global__ void __launch_bounds__(kRankThreads, SP <= 16 ? 4 : 2)
 auroc_lane_config_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
                          uint32_t C, uint32_t N, uint32_t S, bool vec,
                          int64_t *__restrict__ u2_out, int64_t *__restrict__ gt_out,
@@ -251,35 +304,53 @@ auroc_lane_config_kernel(const float *__restrict__ scores, const int8_t *__restr
                          int32_t *status) {
   const int lane = threadIdx.x & 31;
   const uint64_t warps = (uint64_t)gridDim.x * kRankWarps;
+  const bool narrow = (uint64_t)N * (SP * SP / 2) < (1ull << 32);
   bool saw_nan = false;
   for (uint64_t c = (uint64_t)blockIdx.x * kRankWarps + (threadIdx.x >> 5); c < C; c += warps) {
-    long long total = 0, valid = 0, pmin = LLONG_MAX, pmax = -1;
-    for (uint32_t n = lane; n < N; n += 32) {
-      const uint64_t o = c * N + n;
-      long long g, e;
-      int nm, nb;
-      lane_counts<SP>(scores, labels, o, S, vec, g, e, nm, nb, saw_nan);
-      const long long u2 = 2 * g + e;
+    // per-lane sums; 32-bit when no configuration total can reach 2^32
+    // (a canary's 2U is at most 2 (SP/2)^2)
+    uint32_t t32 = 0u, valid = 0u, pmin = 0xFFFFFFFFu, pmax = 0u;
+    unsigned long long t64 = 0ull;
+    auto record = [&](const LaneRow<SP> &r, uint64_t o) {
+      int g, e, nm, nb;
+      lane_rank<SP>(r, g, e, nm, nb, saw_nan);
+      const uint32_t u2 = 2u * (uint32_t)g + (uint32_t)e;
       u2_out[o] = u2;
       if (gt_out) gt_out[o] = g;
       if (eq_out) eq_out[o] = e;
-      const long long pairs = (long long)nm * nb;
+      const uint32_t pairs = (uint32_t)nm * (uint32_t)nb;
       if (pairs > 0) {
-        total += u2;
-        valid += 1;
+        if (narrow) t32 += u2;
+        else t64 += u2;
+        valid += 1u;
         pmin = min(pmin, pairs);
         pmax = max(pmax, pairs);
       }
+    };
+    // two canaries per lane per round, both loaded before either is ranked
+    for (uint32_t n = lane; n < N; n += 64) {
+      const uint64_t o = c * N + n;
+      const bool two = n + 32 < N;
+      LaneRow<SP> ra, rb;
+      lane_load<SP>(scores, labels, o, S, vec, ra);
+      if (two) lane_load<SP>(scores, labels, o + 32, S, vec, rb);
+      record(ra, o);
+      if (two) record(rb, o + 32);
     }
+    valid = __reduce_add_sync(0xFFFFFFFFu, valid);
+    pmin = __reduce_min_sync(0xFFFFFFFFu, pmin);
+    pmax = __reduce_max_sync(0xFFFFFFFFu, pmax);
+    long long total;
+    if (narrow) {
+      total = (long long)__reduce_add_sync(0xFFFFFFFFu, t32);
+    } else {
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      total += __shfl_xor_sync(0xFFFFFFFFu, total, off);
-      valid += __shfl_xor_sync(0xFFFFFFFFu, valid, off);
-      pmin = min(pmin, __shfl_xor_sync(0xFFFFFFFFu, pmin, off));
-      pmax = max(pmax, __shfl_xor_sync(0xFFFFFFFFu, pmax, off));
+      for (int off = 16; off > 0; off >>= 1) t64 += __shfl_xor_sync(0xFFFFFFFFu, t64, off);
+      total = (long long)t64;
     }
     __syncwarp();   // every lane's u2 writes are visible to lane 0 below
-    if (lane == 0) auroc[c] = combine_auroc(labels, c, N, S, u2_out, total, valid, pmin, pmax);
+    if (lane == 0)
+      auroc[c] = combine_auroc(labels, c, N, S, u2_out, total, valid, pmin, pmax);
     __syncwarp();
   }
   if (__any_sync(0xFFFFFFFFu, saw_nan) && lane == 0 && status)
@@ -601,7 +672,7 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
     const int SP = S <= 4 ? 4 : S <= 8 ? 8 : S <= 16 ? 16 : 32;
     // 16-byte row loads only when a row is exactly SP scores and 16-byte aligned
     const bool vec = (S == (uint32_t)SP) && ((uintptr_t)scores % 16 == 0) &&
-                     ((uintptr_t)labels % 4 == 0);
+                     ((uintptr_t)labels % (SP < 16 ? SP : 16) == 0);
     if (many) {
       const uint64_t grid = ((uint64_t)C + kRankWarps - 1) / kRankWarps;   // a warp each
 #define CG_LANE_CONFIG(P)                                                                     \
