@@ -53,6 +53,28 @@ def test_auroc_nonuniform_pairs_bit_exact(cg, orc):
     assert np.isnan(g["auroc"][2]) and np.isnan(o["auroc"][2])
 
 
+@pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
+    (2437, 37, 10, 2, 1, 4), (2440, 64, 32, 3, 2, None), (2500, 33, 4, 1, 0, 3),
+    (2448, 70, 8, 2, 0, None), (2433, 64, 16, 1, 0, 2), (2436, 129, 16, 2, 1, None),
+])
+def test_auroc_batched_lanes_match_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
+    """Batches large enough for the warp-per-8-configurations kernel: partial
+    last batch, canary counts that are not a multiple of 64, every SP,
+    row-aligned and unaligned loads, ties, excluded stages, non-uniform pair
+    counts and a configuration without any pair."""
+    scores, labels = SI.score_arrays(C, N, S, seed=C + 3 * N + S, n_malicious=n_mal,
+                                     tie_levels=ties, excluded=excluded)
+    labels[5, ::3, :] = np.where(labels[5, ::3, :] == 0, -1, labels[5, ::3, :])   # fewer pairs
+    labels[9, :, :] = 0                                                           # no pair
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    for k in ("u2", "gt", "eq"):
+        assert np.array_equal(g[k], o[k]), k
+    fin = ~np.isnan(o["auroc"])
+    assert not fin[9] and np.isnan(g["auroc"][9])
+    assert np.array_equal(g["auroc"][fin].view(np.uint64), o["auroc"][fin].view(np.uint64))
+
+
 def test_auroc_stress_batch(cg, orc):
     """65,536 configurations x 64 canaries x 16 stages."""
     rng = np.random.Generator(np.random.PCG64(5))
