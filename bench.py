@@ -612,40 +612,68 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
 STUDY_METRIC = "AUROC configs/sec (whole study: generate, score and rank every configuration)"
 
 
-def study_pass(cg, torch, configs, dev, bufs, res, drift_events=None):
+def study_pass(cg, torch, configs, dev, bufs, res, drift_events=None, overlap=True):
     """Every configuration of a study on the device: generate, drift scores,
     control labels, per-canary AUROC of rel_l2 / max_abs / cos_dev and of the
-    control, pooled AUROC of rel_l2.  res[c] = those five A-hat values."""
+    control, pooled AUROC of rel_l2.  res[c] = those five A-hat values.
+
+    overlap: configuration c + 1 is generated on one stream while c is scored
+    on another, in alternating pipeline buffers (the generator is bound by
+    integer/FP32 issue, the scoring by HBM, and the generator leaves room on
+    every SM for a drift block).  The passes fork from and join back into the
+    current stream, so a CUDA graph capture of a pass holds both streams."""
+    main = torch.cuda.current_stream()
+    if overlap:
+        s_gen, s_score = bufs["s_gen"], bufs["s_score"]
+        s_gen.wait_stream(main)
+        s_score.wait_stream(main)
+    else:
+        s_gen = s_score = main
     for c, cfg in enumerate(configs):
         S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
         E = S * N * L
+        b = c % 2 if overlap else 0
         desc = cg.PipelineDesc.from_config(cfg)
-        acts = bufs["acts"][:E].view(S, N, L)
-        refs = bufs["refs"][:E].view(S, N, L)
-        labels = bufs["labels"][:N * S].view(1, N, S)
+        acts = bufs["acts"][b][:E].view(S, N, L)
+        refs = bufs["refs"][b][:E].view(S, N, L)
+        labels = bufs["labels"][b][:N * S].view(1, N, S)
         ctrl = bufs["ctrl"][:N * S].view(1, N, S)
-        if cfg.get("gain", 0.0):
-            cg.cg_generate_propagating(desc, cfg["gain"], acts, refs, labels[0], bufs["gws"],
-                                       status=bufs["status"])
-        else:
-            cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"],
-                                    status=bufs["status"])
-        scores = bufs["scores"][:3 * N * S].view(3, N, S)
-        if drift_events is not None:
-            drift_events[c][0].record()
-        cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"], status=bufs["status"])
-        if drift_events is not None:
-            drift_events[c][1].record()
-        cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
-                                  status=bufs["status"])
-        u2 = bufs["u2"][:N].view(1, N)
-        for k in range(3):
-            cg.cg_auroc(scores[k].view(1, N, S), labels, u2=u2, auroc=res[c, k:k + 1],
-                        want_counts=False, status=bufs["status"])
-        cg.cg_auroc(scores[0].view(1, N, S), ctrl, u2=u2, auroc=res[c, 3:4], want_counts=False,
-                    status=bufs["status"])
-        cg.cg_auroc_pooled(scores[0].view(1, N, S), labels, u2=bufs["pu2"], n_mal=bufs["pnm"],
-                           n_ben=bufs["pnb"], auroc=res[c, 4:5], status=bufs["status"])
+        with torch.cuda.stream(s_gen):
+            if overlap and c >= 2:
+                s_gen.wait_event(bufs["scored"][b])      # buffer b is free once c - 2 is scored
+            if cfg.get("gain", 0.0):
+                cg.cg_generate_propagating(desc, cfg["gain"], acts, refs, labels[0], bufs["gws"],
+                                           status=bufs["status"])
+            else:
+                cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"],
+                                        status=bufs["status"])
+            if overlap:
+                bufs["generated"][b].record(s_gen)
+        with torch.cuda.stream(s_score):
+            if overlap:
+                s_score.wait_event(bufs["generated"][b])
+            scores = bufs["scores"][:3 * N * S].view(3, N, S)
+            if drift_events is not None:
+                drift_events[c][0].record(s_score)
+            cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"],
+                               status=bufs["status"])
+            if drift_events is not None:
+                drift_events[c][1].record(s_score)
+            cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
+                                      status=bufs["status"])
+            u2 = bufs["u2"][:N].view(1, N)
+            for k in range(3):
+                cg.cg_auroc(scores[k].view(1, N, S), labels, u2=u2, auroc=res[c, k:k + 1],
+                            want_counts=False, status=bufs["status"])
+            cg.cg_auroc(scores[0].view(1, N, S), ctrl, u2=u2, auroc=res[c, 3:4], want_counts=False,
+                        status=bufs["status"])
+            cg.cg_auroc_pooled(scores[0].view(1, N, S), labels, u2=bufs["pu2"], n_mal=bufs["pnm"],
+                               n_ben=bufs["pnb"], auroc=res[c, 4:5], status=bufs["status"])
+            if overlap:
+                bufs["scored"][b].record(s_score)
+    if overlap:
+        main.wait_stream(s_gen)
+        main.wait_stream(s_score)
 
 
 def run_study(args, ranks: Ranks):
@@ -664,9 +692,14 @@ def run_study(args, ranks: Ranks):
     dws = max(cg.cg_drift_workspace_size(c["n_shards"], c["n_canaries"],
                                          c["tokens"] * c["hidden"]) for c in configs)
     bufs = {
-        "acts": torch.empty(maxE, dtype=torch.float16, device=dev),
-        "refs": torch.empty(maxE, dtype=torch.float32, device=dev),
-        "labels": torch.empty(maxNS, dtype=torch.int8, device=dev),
+        # two pipeline buffers: one being generated while the other is scored
+        "acts": [torch.empty(maxE, dtype=torch.float16, device=dev) for _ in range(2)],
+        "refs": [torch.empty(maxE, dtype=torch.float32, device=dev) for _ in range(2)],
+        "labels": [torch.empty(maxNS, dtype=torch.int8, device=dev) for _ in range(2)],
+        "s_gen": torch.cuda.Stream(device=dev),
+        "s_score": torch.cuda.Stream(device=dev),
+        "generated": [torch.cuda.Event() for _ in range(2)],
+        "scored": [torch.cuda.Event() for _ in range(2)],
         "ctrl": torch.empty(maxNS, dtype=torch.int8, device=dev),
         "scores": torch.empty(3 * maxNS, dtype=torch.float32, device=dev),
         "u2": torch.empty(maxN, dtype=torch.int64, device=dev),
@@ -725,10 +758,15 @@ def run_study(args, ranks: Ranks):
         raise RuntimeError(f"device status {word} during the study")
     # one more pass with events around every drift call: the drift reduction's
     # own bandwidth on these pipelines (6 algorithmic bytes per element)
+    # (one stream, nothing overlapping it); its A-hat values must equal the
+    # overlapped passes' bit for bit
     dev_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in configs]
-    study_pass(cg, torch, configs, dev, bufs, res, drift_events=dev_ev)
+    overlapped_res = res.clone()
+    study_pass(cg, torch, configs, dev, bufs, res, drift_events=dev_ev, overlap=False)
     torch.cuda.synchronize()
+    if not torch.equal(res.view(torch.int64), overlapped_res.view(torch.int64)):
+        raise RuntimeError("the overlapped passes' A-hat values differ from the one-stream pass")
     drift_ms = sum(a.elapsed_time(b) for a, b in dev_ev)
     drift_bytes = float(sum(SI.n_elements(c) for c in configs)) * BYTES_PER_ELEMENT
     peak, peak_kind = measured_peaks()
@@ -753,7 +791,8 @@ def run_study(args, ranks: Ranks):
         "config": {"workload": f"study '{args.study}': {len(configs)} configurations",
                    "elements_per_pass": elems,
                    "step": "per configuration: generate (2 to 4 kernels), drift (2), control labels, "
-                           "3 + 1 per-canary AUROC, 1 pooled AUROC"},
+                           "3 + 1 per-canary AUROC, 1 pooled AUROC; configuration c + 1 is generated "
+                           "on a second stream while c is scored (two pipeline buffers)"},
         "elements_per_s": elems / (ms / 1e3),
         "execution": "CUDA graph of one whole pass, replayed" if graph is not None else "eager",
         "eager": {"value": total_cfg / (ms_eager / 1e3), "unit": "configs/s",

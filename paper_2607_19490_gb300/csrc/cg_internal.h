@@ -51,6 +51,7 @@ cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32
 // ---------------------------------------------------------------- generator
 constexpr uint32_t kGenStatChunk = 65536;   // elements per statistics work item
 constexpr int kGenThreads = 256;
+constexpr int kGenBlocksPerSm = 3;          // leaves room for a co-running drift block
 constexpr uint32_t kMaxShards = 1024;
 constexpr uint32_t kMaxOutliers = 256;
 

@@ -712,12 +712,18 @@ cudaError_t launch_box_muller_pairs(const uint32_t *words, uint64_t n_pairs, flo
   return cudaGetLastError();
 }
 
+// Generator blocks per SM: the occupancy of pass 1, capped at kGenBlocksPerSm
+// so that one drift block (288 threads x 32 registers, 147 KB of shared
+// memory) still fits beside them.  A caller that scores one configuration
+// while it generates the next on another stream then overlaps the two: the
+// generator is bound by integer/FP32 issue, the drift reduction by HBM.  At
+// 4 blocks per SM instead of 3 the generator alone is about 3 % faster.
 int gen_occupancy() {
   int n = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_refs_kernel<true>, kGenThreads, 0) !=
       cudaSuccess)
     return 0;
-  return n;
+  return n < kGenBlocksPerSm ? n : kGenBlocksPerSm;
 }
 
 }  // namespace cg
