@@ -110,20 +110,12 @@ __device__ __forceinline__ float2 box_muller(uint32_t x0, uint32_t x1) {
   return make_float2(r * cs.x, r * cs.y);
 }
 
-// The four normals of one Philox block from precomputed round keys.
+// The four normals of one Philox block from precomputed round keys (counter
+// word 3 = c3: 0 for every live draw, the replica index for an independent
+// benign recompute).
 __device__ __forceinline__ float4 normals4_rk(const PhiloxRoundKeys &rk, uint32_t q, uint32_t c1,
                                               uint32_t c2, uint32_t c3 = 0u) {
   const uint4 w = philox4x32_10_rk(make_uint4(q, c1, c2, c3), rk);
-  const float2 a = box_muller(w.x, w.y);
-  const float2 b = box_muller(w.z, w.w);
-  return make_float4(a.x, a.y, b.x, b.y);
-}
-
-// The four normals of one Philox block (counter word 3 = c3: 0 for every
-// live draw, the replica index for an independent benign recompute).
-__device__ __forceinline__ float4 normals4(uint2 key, uint32_t q, uint32_t c1, uint32_t c2,
-                                           uint32_t c3 = 0u) {
-  const uint4 w = philox4x32_10(make_uint4(q, c1, c2, c3), key);
   const float2 a = box_muller(w.x, w.y);
   const float2 b = box_muller(w.z, w.w);
   return make_float4(a.x, a.y, b.x, b.y);
