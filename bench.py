@@ -518,6 +518,24 @@ def auroc_batches(cg, torch, dev, stream):
         ms = e0.elapsed_time(e1) / reps
         out[f"{name}_configs_per_s"] = C / (ms / 1e3)
         out[f"{name}_ms"] = ms
+        if name == "stress_batch":
+            # the pooled Mann-Whitney (f2): one block-wide bitonic sort of the
+            # N * S labelled scores per configuration
+            pu = {k: torch.empty((C,), dtype=torch.int64, device=dev) for k in ("u2", "nm", "nb")}
+            pa = torch.empty((C,), dtype=torch.float64, device=dev)
+            for _ in range(3):
+                cg.cg_auroc_pooled(scores, labels, u2=pu["u2"], n_mal=pu["nm"], n_ben=pu["nb"],
+                                   auroc=pa)
+            e0.record(stream)
+            for _ in range(reps):
+                cg.cg_auroc_pooled(scores, labels, u2=pu["u2"], n_mal=pu["nm"], n_ben=pu["nb"],
+                                   auroc=pa)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            pms = e0.elapsed_time(e1) / reps
+            out["pooled_stress_batch_configs_per_s"] = C / (pms / 1e3)
+            out["pooled_stress_batch_ms"] = pms
+            out["pooled_stress_batch_read_GBps"] = C * N * S * 5 / (pms / 1e3) / 1e9
         del scores, labels
     return out
 

@@ -514,7 +514,7 @@ __global__ void control_labels_kernel(const int8_t *__restrict__ labels, uint32_
 // bitonic network sorts them, and every malicious key adds twice its
 // midrank, lo + 1 + hi, where [lo, hi) is the run of its score found by
 // binary search.  2U = sum(2 midrank) - n_mal (n_mal + 1), exact in int64.
-constexpr int kPoolThreads = 1024;
+constexpr int kPoolThreads = 256;
 constexpr int kPoolWarps = kPoolThreads / 32;
 
 __device__ __forceinline__ uint32_t order_key(float x) {
@@ -523,98 +523,163 @@ __device__ __forceinline__ uint32_t order_key(float x) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-__device__ __forceinline__ uint32_t lower_bound_u64(const unsigned long long *k, uint32_t n,
-                                                    unsigned long long v) {
-  uint32_t lo = 0, hi = n;
-  while (lo < hi) {
-    const uint32_t mid = (lo + hi) >> 1;
-    if (k[mid] < v) lo = mid + 1;
-    else hi = mid;
+// First index of the sorted, padded k[0, M) (M a power of two; the padding
+// key 0xFFFFFFFF is above every score's key) whose key is >= v (lower) or
+// > v (upper): log2(M) fixed steps, no divergence.
+__device__ __forceinline__ uint32_t bound_u32(const uint32_t *k, uint32_t M, uint32_t v,
+                                              bool upper) {
+  uint32_t pos = 0;
+  for (uint32_t step = M >> 1; step > 0; step >>= 1) {
+    const uint32_t x = k[pos + step - 1];
+    pos += (upper ? (x <= v) : (x < v)) ? step : 0u;
   }
-  return lo;
+  const uint32_t x = k[pos];
+  return pos + ((upper ? (x <= v) : (x < v)) ? 1u : 0u);
 }
 
+// Bitonic sort of up to 64 keys held by one warp, two per lane (key e at
+// register e / 32 of lane e % 32): stride 32 swaps the lane's registers,
+// smaller strides pair lanes through shuffles.
+__device__ __forceinline__ void warp_sort64(uint32_t &r0, uint32_t &r1, uint32_t M, int lane) {
+  for (uint32_t k = 2; k <= M; k <<= 1) {
+    for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+      if (j == 32) {
+        const bool up = ((uint32_t)lane & k) == 0;          // e = lane, partner lane + 32
+        const uint32_t lo = min(r0, r1), hi = max(r0, r1);
+        r0 = up ? lo : hi;
+        r1 = up ? hi : lo;
+      } else {
+        const uint32_t p0 = __shfl_xor_sync(0xFFFFFFFFu, r0, (int)j);
+        const uint32_t p1 = __shfl_xor_sync(0xFFFFFFFFu, r1, (int)j);
+        const bool lower = ((uint32_t)lane & j) == 0;
+        const bool up0 = ((uint32_t)lane & k) == 0;
+        const bool up1 = (((uint32_t)lane + 32u) & k) == 0;
+        r0 = (lower == up0) ? min(r0, p0) : max(r0, p0);
+        r1 = (lower == up1) ? min(r1, p1) : max(r1, p1);
+      }
+    }
+  }
+}
+
+// Pooled Mann-Whitney (Sec. 3.4), one block per configuration.  The
+// labelled scores become order-preserving 32-bit keys, compacted into
+// shared memory (malicious from the front, benign from the back, warp-
+// aggregated offsets; the order inside each side does not matter).  Only
+// the smaller side is sorted (a block bitonic sort of its padded
+// power-of-two size Ms); every key of the larger side then takes its lower
+// and upper bound in the sorted side, which give its pairs above and tied:
+//   smaller side malicious: gt += #(m > b) = s - upper(b), eq += upper - lower
+//   smaller side benign:    gt += #(b < m) = lower(m),     eq += upper - lower
+// 2U = 2 gt + eq is an exact integer and A-hat = 2U / (2 n_m n_b) one fp64
+// division.  Shared memory: per + Ms 32-bit keys.
 __global__ void __launch_bounds__(kPoolThreads)
 auroc_pooled_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
-                    uint32_t C, uint32_t per, uint32_t M, int64_t *__restrict__ u2_out,
+                    uint32_t C, uint32_t per, uint32_t Ms, int64_t *__restrict__ u2_out,
                     int64_t *__restrict__ nm_out, int64_t *__restrict__ nb_out,
                     double *__restrict__ auroc, int32_t *status) {
-  extern __shared__ unsigned long long keys[];
-  __shared__ unsigned int count;
-  __shared__ long long red[kPoolWarps][3];
+  extern __shared__ uint32_t pool_keys[];
+  uint32_t *sorted = pool_keys + per;
+  __shared__ unsigned int n_mal_s, n_ben_s;
+  __shared__ unsigned long long red[kPoolWarps][2];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  bool nan_seen = false;
   for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
-    if (tid == 0) count = 0u;
+    if (tid == 0) n_mal_s = n_ben_s = 0u;
     __syncthreads();
-    bool nan_seen = false;
     const float *m = scores + (uint64_t)c * per;
     const int8_t *l = labels + (uint64_t)c * per;
-    for (uint32_t i = tid; i < per; i += kPoolThreads) {
-      const int lab = l[i];
-      if (lab != 0 && lab != 1) continue;
-      const float x = m[i];
-      if (is_nan_f(x)) {
-        nan_seen = true;
-        continue;
-      }
-      const unsigned int pos = atomicAdd(&count, 1u);
-      keys[pos] = ((unsigned long long)order_key(x) << 32) | (unsigned long long)lab;
-    }
-    __syncthreads();
-    const uint32_t n = count;
-    for (uint32_t i = n + tid; i < M; i += kPoolThreads) keys[i] = ~0ull;   // pad: sorts last
-    __syncthreads();
-    for (uint32_t k = 2; k <= M; k <<= 1) {
-      for (uint32_t j = k >> 1; j > 0; j >>= 1) {
-        for (uint32_t i = tid; i < M; i += kPoolThreads) {
-          const uint32_t ixj = i ^ j;
-          if (ixj > i) {
-            const unsigned long long a = keys[i], b = keys[ixj];
-            const bool up = (i & k) == 0;
-            if ((a > b) == up) {
-              keys[i] = b;
-              keys[ixj] = a;
-            }
+    for (uint32_t i0 = 0; i0 < per; i0 += kPoolThreads) {
+      const uint32_t i = i0 + tid;
+      int lab = -1;
+      float x = 0.f;
+      if (i < per) {
+        lab = l[i];
+        if (lab == 0 || lab == 1) {
+          x = m[i];
+          if (is_nan_f(x)) {
+            nan_seen = true;
+            lab = -1;
           }
         }
-        __syncthreads();
+      }
+      const uint32_t mal = __ballot_sync(0xFFFFFFFFu, lab == 1);
+      const uint32_t ben = __ballot_sync(0xFFFFFFFFu, lab == 0);
+      uint32_t base_m = 0u, base_b = 0u;
+      if (lane == 0) {
+        if (mal) base_m = atomicAdd(&n_mal_s, (unsigned)__popc(mal));
+        if (ben) base_b = atomicAdd(&n_ben_s, (unsigned)__popc(ben));
+      }
+      base_m = __shfl_sync(0xFFFFFFFFu, base_m, 0);
+      base_b = __shfl_sync(0xFFFFFFFFu, base_b, 0);
+      if (lab == 1) pool_keys[base_m + __popc(mal & lt_mask)] = order_key(x);
+      else if (lab == 0) pool_keys[per - 1u - (base_b + __popc(ben & lt_mask))] = order_key(x);
+    }
+    __syncthreads();
+    const uint32_t nm = n_mal_s, nb = n_ben_s;
+    const bool small_mal = nm <= nb;
+    const uint32_t ns = small_mal ? nm : nb, nl = small_mal ? nb : nm;
+    const uint32_t *small = small_mal ? pool_keys : pool_keys + (per - nb);
+    const uint32_t *large = small_mal ? pool_keys + (per - nb) : pool_keys;
+    uint32_t M = 1;
+    while (M < ns) M <<= 1;
+    if (M <= 64) {
+      // a small side of up to 64 keys: one warp sorts it in registers
+      if (warp == 0) {
+        uint32_t r0 = (uint32_t)lane < ns ? small[lane] : 0xFFFFFFFFu;
+        uint32_t r1 = (uint32_t)lane + 32u < ns ? small[lane + 32] : 0xFFFFFFFFu;
+        warp_sort64(r0, r1, M, lane);
+        if ((uint32_t)lane < M) sorted[lane] = r0;
+        if ((uint32_t)lane + 32u < M) sorted[lane + 32] = r1;
+      }
+      __syncthreads();
+    } else {
+      for (uint32_t i = tid; i < M; i += kPoolThreads) sorted[i] = i < ns ? small[i] : 0xFFFFFFFFu;
+      __syncthreads();
+      for (uint32_t k = 2; k <= M; k <<= 1) {
+        for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+          for (uint32_t i = tid; i < M; i += kPoolThreads) {
+            const uint32_t ixj = i ^ j;
+            if (ixj > i) {
+              const uint32_t a = sorted[i], b = sorted[ixj];
+              if ((a > b) == ((i & k) == 0)) {
+                sorted[i] = b;
+                sorted[ixj] = a;
+              }
+            }
+          }
+          __syncthreads();
+        }
       }
     }
-    long long rs = 0, nm = 0, nb = 0;
-    for (uint32_t i = tid; i < n; i += kPoolThreads) {
-      const unsigned long long v = keys[i];
-      if (v & 1ull) {
-        const unsigned long long hk = v >> 32;
-        const uint32_t lo = lower_bound_u64(keys, n, hk << 32);
-        const uint32_t hi = lower_bound_u64(keys, n, (hk + 1) << 32);
-        rs += (long long)lo + 1 + (long long)hi;
-        nm += 1;
-      } else {
-        nb += 1;
+    unsigned long long gt = 0ull, eq = 0ull;
+    if (ns > 0) {
+      for (uint32_t i = tid; i < nl; i += kPoolThreads) {
+        const uint32_t v = large[i];
+        const uint32_t lo = bound_u32(sorted, M, v, false);
+        const uint32_t hi = bound_u32(sorted, M, v, true);
+        gt += small_mal ? (ns - hi) : lo;
+        eq += hi - lo;
       }
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-      rs += __shfl_down_sync(0xFFFFFFFFu, rs, off);
-      nm += __shfl_down_sync(0xFFFFFFFFu, nm, off);
-      nb += __shfl_down_sync(0xFFFFFFFFu, nb, off);
+      gt += __shfl_down_sync(0xFFFFFFFFu, gt, off);
+      eq += __shfl_down_sync(0xFFFFFFFFu, eq, off);
     }
     if (lane == 0) {
-      red[warp][0] = rs;
-      red[warp][1] = nm;
-      red[warp][2] = nb;
+      red[warp][0] = gt;
+      red[warp][1] = eq;
     }
-    if (__any_sync(0xFFFFFFFFu, nan_seen) && lane == 0 && status)
-      atomicOr(status, CG_DEVFLAG_NAN_SCORE);
     __syncthreads();
     if (tid == 0) {
-      long long R = 0, NM = 0, NB = 0;
+      unsigned long long G = 0ull, E = 0ull;
       for (int w = 0; w < kPoolWarps; ++w) {
-        R += red[w][0];
-        NM += red[w][1];
-        NB += red[w][2];
+        G += red[w][0];
+        E += red[w][1];
       }
-      const long long u2 = R - NM * (NM + 1);
+      const long long u2 = (long long)(2ull * G + E);
+      const long long NM = nm, NB = nb;
       u2_out[c] = u2;
       if (nm_out) nm_out[c] = NM;
       if (nb_out) nb_out[c] = NB;
@@ -622,6 +687,8 @@ auroc_pooled_kernel(const float *__restrict__ scores, const int8_t *__restrict__
     }
     __syncthreads();
   }
+  if (__any_sync(0xFFFFFFFFu, nan_seen) && lane == 0 && status)
+    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
 }  // namespace
@@ -633,18 +700,24 @@ cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint3
   DeviceInfo info;
   if (!device_info(&info)) return cudaGetLastError();
   const uint32_t per = N * S;
-  uint32_t M = 2;
-  while (M < per) M <<= 1;
-  const size_t smem = (size_t)M * sizeof(unsigned long long);
+  uint32_t Ms = 1;                                // the smaller side holds at most per / 2 keys
+  while (Ms < (per + 1) / 2) Ms <<= 1;
+  const size_t smem = (size_t)(per + Ms) * sizeof(uint32_t);
   cudaError_t err = cudaFuncSetAttribute(auroc_pooled_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
-  uint64_t per_sm = smem > 0 ? (200u * 1024u) / (smem + 1024) : 1;
-  if (per_sm < 1) per_sm = 1;
-  uint64_t grid = (uint64_t)info.sm_count * per_sm;
-  if (grid > C) grid = C;
-  auroc_pooled_kernel<<<(unsigned)grid, kPoolThreads, smem, stream>>>(scores, labels, C, per, M, u2,
-                                                                      n_mal, n_ben, auroc, status);
+  uint64_t grid = C;
+  if (C > (uint32_t)info.sm_count) {
+    int occ = 0;
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, auroc_pooled_kernel, kPoolThreads,
+                                                        smem);
+    if (err != cudaSuccess) return err;
+    const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)(occ > 0 ? occ : 1);
+    if (grid > resident) grid = resident;
+  }
+  auroc_pooled_kernel<<<(unsigned)grid, kPoolThreads, smem, stream>>>(scores, labels, C, per, Ms,
+                                                                      u2, n_mal, n_ben, auroc,
+                                                                      status);
   return cudaGetLastError();
 }
 

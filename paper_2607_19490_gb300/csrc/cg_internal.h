@@ -99,7 +99,7 @@ constexpr uint32_t kMaxRankShards = 1024;
 cudaError_t launch_control_labels(const int8_t *labels, uint32_t C, uint32_t N, uint32_t S,
                                   uint64_t seed, uint32_t config_id0, int8_t *ctrl,
                                   int32_t *status, cudaStream_t stream);
-constexpr uint32_t kMaxPooled = 16384;   // labelled scores per configuration (128 KiB of keys)
+constexpr uint32_t kMaxPooled = 16384;   // labelled scores per configuration (96 KiB of keys)
 cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint32_t C,
                                 uint32_t N, uint32_t S, int64_t *u2, int64_t *n_mal,
                                 int64_t *n_ben, double *auroc, int32_t *status,
