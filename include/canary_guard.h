@@ -284,6 +284,9 @@ cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs,
  *   different streams or from different host threads) race and corrupt
  *   each other's results; serialise them on one stream.  Nothing in it
  *   needs to start at zero: every partial is written before it is read.
+ *   d_status is checked for alignment and otherwise unused: this path runs
+ *   the register-streaming kernel, which has no wait that could give up
+ *   (a NaN element shows in the scores, as with cg_drift_scores).
  */
 #define CG_NOALLOC_CHUNK_ELEMENTS 16384u
 #define CG_NOALLOC_MAX_WORK_ITEMS 262144u

@@ -341,7 +341,7 @@ cg_status cg_drift_scores_noalloc(const uint16_t *d_acts, const float *d_refs,
   if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || !aligned(d_scores, 4) ||
       (d_status && !aligned(d_status, 4)))
     return CG_ERR_ALIGNMENT;
-  (void)d_status;
+  (void)d_status;   // the register-streaming kernel has no wait that could give up
   return from_cuda(cg::launch_drift_noalloc(d_acts, d_refs, n_shards, n_canaries, seg_len,
                                             d_scores, stat_stride, (cudaStream_t)stream));
 }
