@@ -3,8 +3,10 @@
 // plus the labels of the scrambled-label negative control (Sec. 4.5).
 //
 // S <= 32: one lane per canary -- auroc_lane_config_kernel (many
-// configurations: a warp per configuration) or auroc_lane_canary_kernel +
-// auroc_config_kernel (few: lanes over all canaries, then a combine).
+// configurations: a warp per configuration), auroc_block_kernel (few
+// configurations of at most 1024 canaries: a block per configuration, one
+// launch) or auroc_lane_canary_kernel + auroc_config_kernel (few, more
+// canaries: lanes over all canaries, then a combine).
 // S > 32: one warp per canary with the stages strided over the lanes
 // (auroc_kernel / auroc_canary_kernel).
 // Counts are integers (exact in any order); the configuration's A-hat is
@@ -374,6 +376,69 @@ auroc_lane_canary_kernel(const float *__restrict__ scores, const int8_t *__restr
     if (eq_out) eq_out[o] = e;
   }
   if (saw_nan && status) atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+}
+
+// Few configurations of at most kBlockRankCanaries canaries: one block per
+// configuration ranks its canaries (a thread per canary, lane_counts) and
+// combines them itself, so a single-configuration call is one launch.
+constexpr uint32_t kBlockRankCanaries = 1024;
+
+template <int SP>
+__global__ void __launch_bounds__(kRankThreads)
+auroc_block_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels, uint32_t C,
+                   uint32_t N, uint32_t S, bool vec, int64_t *__restrict__ u2_out,
+                   int64_t *__restrict__ gt_out, int64_t *__restrict__ eq_out,
+                   double *__restrict__ auroc, int32_t *status) {
+  __shared__ unsigned long long red_total[kRankWarps];
+  __shared__ uint32_t red_small[kRankWarps][3];   // valid, pmin, pmax
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  bool saw_nan = false;
+  for (uint32_t c = blockIdx.x; c < C; c += gridDim.x) {
+    unsigned long long total = 0ull;
+    uint32_t valid = 0u, pmin = 0xFFFFFFFFu, pmax = 0u;
+    for (uint32_t n = tid; n < N; n += kRankThreads) {
+      const uint64_t o = (uint64_t)c * N + n;
+      long long g, e;
+      int nm, nb;
+      lane_counts<SP>(scores, labels, o, S, vec, g, e, nm, nb, saw_nan);
+      const long long u2 = 2 * g + e;
+      u2_out[o] = u2;
+      if (gt_out) gt_out[o] = g;
+      if (eq_out) eq_out[o] = e;
+      const uint32_t pairs = (uint32_t)nm * (uint32_t)nb;
+      if (pairs > 0) {
+        total += (unsigned long long)u2;
+        valid += 1u;
+        pmin = min(pmin, pairs);
+        pmax = max(pmax, pairs);
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) total += __shfl_xor_sync(0xFFFFFFFFu, total, off);
+    valid = __reduce_add_sync(0xFFFFFFFFu, valid);
+    pmin = __reduce_min_sync(0xFFFFFFFFu, pmin);
+    pmax = __reduce_max_sync(0xFFFFFFFFu, pmax);
+    if (lane == 0) {
+      red_total[warp] = total;
+      red_small[warp][0] = valid;
+      red_small[warp][1] = pmin;
+      red_small[warp][2] = pmax;
+    }
+    __syncthreads();   // also makes every thread's u2 writes visible to thread 0
+    if (tid == 0) {
+      unsigned long long T = 0ull;
+      uint32_t V = 0u, lo = 0xFFFFFFFFu, hi = 0u;
+      for (int w = 0; w < kRankWarps; ++w) {
+        T += red_total[w];
+        V += red_small[w][0];
+        lo = min(lo, red_small[w][1]);
+        hi = max(hi, red_small[w][2]);
+      }
+      auroc[c] = combine_auroc(labels, c, N, S, u2_out, (long long)T, V, lo, hi);
+    }
+    __syncthreads();
+  }
+  if (__syncthreads_or(saw_nan) && tid == 0 && status) atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
 // Small batches (few configurations): the same per-canary counts with one
@@ -759,6 +824,20 @@ cudaError_t launch_auroc(const float *scores, const int8_t *labels, uint32_t C, 
         default: CG_LANE_CONFIG(32); break;
       }
 #undef CG_LANE_CONFIG
+      return cudaGetLastError();
+    }
+    if (N <= kBlockRankCanaries) {
+      // few configurations of few canaries: one block each, one launch
+#define CG_BLOCK_RANK(P)                                                                     \
+  auroc_block_kernel<P><<<C, kRankThreads, 0, stream>>>(scores, labels, C, N, S, vec, u2, gt, eq, \
+                                                       auroc, status)
+      switch (SP) {
+        case 4: CG_BLOCK_RANK(4); break;
+        case 8: CG_BLOCK_RANK(8); break;
+        case 16: CG_BLOCK_RANK(16); break;
+        default: CG_BLOCK_RANK(32); break;
+      }
+#undef CG_BLOCK_RANK
       return cudaGetLastError();
     }
     uint64_t blocks = (total + kRankThreads - 1) / kRankThreads;

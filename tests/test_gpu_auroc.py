@@ -29,7 +29,7 @@ def run(cg, scores, labels, status=None):
 @pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
     (1, 1, 2, 1, 0, None), (5, 7, 4, 1, 0, None), (3, 64, 16, 1, 0, 3), (4, 9, 32, 3, 2, 5),
     (2, 5, 33, 2, 0, 4), (2, 3, 100, 7, 5, None), (1, 2, 1024, 10, 3, 6), (324, 64, 16, 1, 0, None),
-    (6, 300, 8, 2, 1, 2),
+    (6, 300, 8, 2, 1, 2), (2, 1500, 8, 2, 1, 3), (1, 4097, 16, 3, 2, None),
 ])
 def test_auroc_matches_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
     scores, labels = SI.score_arrays(C, N, S, seed=C + N + S, n_malicious=n_mal,
