@@ -150,3 +150,27 @@ def test_pooled_nan_flag(cg, orc):
     o = orc.auroc_pooled(scores, labels, allow_nan=True)
     assert cg.cg_read_status(st)[0] == 4
     assert np.array_equal(g["u2"].cpu().numpy(), o["u2"])
+
+
+@pytest.mark.parametrize("C,N,S", [(2, 5, 8), (400, 8, 16), (2, 3, 40), (320, 33, 4)],
+                         ids=["block", "lane_config", "wide", "lane_config_S4"])
+def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
+    """A NaN score on a stage the labels exclude (-1) is not part of any pair:
+    no NaN flag, and counts and A-hat equal the oracle's, on every kernel
+    path (per-canary and pooled)."""
+    import torch
+    scores, labels = SI.score_arrays(C, N, S, seed=C + N + S, n_malicious=1, excluded=2)
+    scores[labels == -1] = np.nan
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = run(cg, scores, labels, status=st)
+    o = orc.auroc(scores, labels)
+    assert cg.cg_read_status(st) == (0, 0)
+    for k in ("u2", "gt", "eq"):
+        assert np.array_equal(g[k], o[k]), k
+    assert np.array_equal(g["auroc"].view(np.uint64), o["auroc"].view(np.uint64))
+    gp = cg.cg_auroc_pooled(torch.from_numpy(scores).cuda(), torch.from_numpy(labels).cuda(),
+                            status=st)
+    op = orc.auroc_pooled(scores, labels)
+    assert cg.cg_read_status(st) == (0, 0)
+    assert np.array_equal(gp["u2"].cpu().numpy(), op["u2"])
+    assert np.array_equal(gp["auroc"].cpu().numpy().view(np.uint64), op["auroc"].view(np.uint64))
