@@ -215,9 +215,12 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * d_scores[stat * stat_stride + n * S + s] (stat_stride >= N * S; pass
  * N * S for a dense [3][N][S] block).  Each element of d_acts and d_refs is
  * read once from HBM.  Sums are accumulated in fp32 per chunk of 16384
- * elements and combined in fp64, so element magnitudes must stay below
- * about 1e17 for the squared sums to remain finite.  d_ws: >= cg_drift_workspace_size bytes, 16-byte
- * aligned, scratch.
+ * elements and combined in fp64, so finite element magnitudes must stay
+ * below about 1e17 for the squared sums to remain finite.  A NaN element
+ * makes rel_l2 and cos_dev NaN (max_abs skips it); an infinite live
+ * element (fp16 +-inf, which an untrusted hop may send) makes rel_l2 and
+ * max_abs +inf and cos_dev NaN.  d_ws: >= cg_drift_workspace_size bytes,
+ * 16-byte aligned, scratch.
  */
 cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
                           uint32_t n_shards, uint32_t n_canaries,

@@ -203,6 +203,8 @@ drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_s
   const double H = A + E;
   if (isnan(D) || isnan(E) || isnan(A)) {
     cosd = NAN;
+  } else if (H > 0.0 && A > 0.0 && (isinf(D) || isinf(E))) {
+    cosd = NAN;                                  // an infinite live element: h / |h| is inf / inf
   } else if (H > 0.0 && A > 0.0) {
     const float sh = sqrtf((float)H), sa = sqrtf((float)A);
     const float gap = (float)E / (sh + sa);

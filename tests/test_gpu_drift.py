@@ -189,3 +189,28 @@ def test_drift_bulk_full_size_matches_stream(cg, algo):
     assert np.array_equal(a[1], b[1])
     del acts, refs
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("algo", [1, 2])
+def test_drift_infinite_and_extreme_live_values(cg, orc, algo):
+    """Live values an untrusted hop may send: +inf and -inf (rel_l2 and
+    max_abs +inf, cos_dev NaN), the largest finite fp16 (65504) and fp16
+    subnormals, against the oracle on the same bytes."""
+    import torch
+    S, N, L = 2, 4, 4096
+    acts, refs = SI.drift_arrays(S, N, L, seed=31)
+    h = acts.view(np.float16).copy()
+    h[0, 1, 17] = np.inf                       # one +inf element
+    h[0, 2, 5] = -np.inf                       # one -inf element
+    h[0, 3, 100] = np.inf                      # +inf and -inf in one segment
+    h[0, 3, 200] = -np.inf
+    h[1, 0, :8] = np.float16(65504.0)          # the largest finite fp16
+    h[1, 1, :] = np.float16(6.0e-8)            # subnormal fp16 everywhere
+    h[1, 2, ::3] = np.float16(-1.0e-6)         # a mix of subnormals
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = run(cg, h.view(np.uint16), refs, S, N, algo=algo, status=st).cpu().numpy()
+    o = orc.drift_scores(h.view(np.uint16), refs, S, N)
+    assert cg.cg_read_status(st) == (0, 0)
+    assert_scores_close(g, o, what=f"algo {algo}")
+    for n in (1, 2, 3):
+        assert np.isinf(g[0, n, 0]) and np.isinf(g[1, n, 0]) and np.isnan(g[2, n, 0])
