@@ -174,3 +174,22 @@ def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
     assert cg.cg_read_status(st) == (0, 0)
     assert np.array_equal(gp["u2"].cpu().numpy(), op["u2"])
     assert np.array_equal(gp["auroc"].cpu().numpy().view(np.uint64), op["auroc"].view(np.uint64))
+
+
+@pytest.mark.parametrize("C,N,S", [(3, 40, 8), (400, 8, 16), (2, 6, 40)],
+                         ids=["block", "lane_config", "wide"])
+def test_auroc_infinities_and_signed_zero(cg, orc, C, N, S):
+    """Scores of +inf (a drift score of an infinite activation), -inf, +0 and
+    -0 (equal, a tie) among finite ones: counts and A-hat equal the oracle's
+    on every per-canary path."""
+    scores, labels = SI.score_arrays(C, N, S, seed=C * 3 + N + S, n_malicious=2, excluded=1,
+                                     tie_levels=4)
+    rng = np.random.Generator(np.random.PCG64(C + S))
+    specials = np.array([np.inf, -np.inf, 0.0, -0.0], np.float32)
+    pick = rng.random(scores.shape) < 0.2
+    scores[pick] = specials[rng.integers(0, 4, size=int(pick.sum()))]
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    for k in ("u2", "gt", "eq"):
+        assert np.array_equal(g[k], o[k]), k
+    assert np.array_equal(g["auroc"].view(np.uint64), o["auroc"].view(np.uint64))

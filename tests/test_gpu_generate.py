@@ -74,6 +74,8 @@ CASES = {
     "snr_step": SI.shrink(SI.snr_configs()[5], n_canaries=3, tokens=4, hidden=1024),
     "signflip_full": SI.shrink(SI.TINY, tamper=SI.TAMPER_SIGNFLIP_FULL, malicious=(0, 3)),
     "scale": SI.shrink(SI.TINY, tamper=SI.TAMPER_SCALE, tamper_param=1.1),
+    "scale_overflow": SI.shrink(SI.TINY, tamper=SI.TAMPER_SCALE, tamper_param=1.0e5),
+    "scale_subnormal": SI.shrink(SI.TINY, tamper=SI.TAMPER_SCALE, tamper_param=1.0e-6),
     "collusion": SI.shrink(SI.TINY, n_shards=8, malicious=(1, 3, 5, 7), noise=SI.NOISE_PAPER),
     "ragged_d100": SI.shrink(SI.TINY, hidden=100, tokens=3, n_outlier=3),
     "ragged_L7": SI.shrink(SI.TINY, hidden=7, tokens=1, n_outlier=1,
