@@ -118,7 +118,7 @@ def test_control_no_benign_flag(cg):
 @pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
     (1, 1, 2, 1, 0, None), (5, 7, 4, 1, 0, None), (3, 64, 16, 1, 0, 3), (4, 9, 32, 3, 2, 5),
     (2, 256, 16, 1, 0, None), (2, 1000, 16, 2, 1, 7), (324, 64, 16, 1, 0, None), (1, 1, 1000, 10, 3, 6),
-    (6, 50, 4, 3, 0, 3), (1, 1024, 16, 9, 0, 4), (1000, 32, 8, 5, 1, 3),
+    (6, 50, 4, 3, 0, 3), (1, 1024, 16, 9, 0, 4), (1000, 32, 8, 5, 1, 3), (2, 16, 8, 2, 0, 1),
 ])
 def test_pooled_matches_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
     import torch

@@ -207,6 +207,8 @@ def test_drift_infinite_and_extreme_live_values(cg, orc, algo):
     h[1, 0, :8] = np.float16(65504.0)          # the largest finite fp16
     h[1, 1, :] = np.float16(6.0e-8)            # subnormal fp16 everywhere
     h[1, 2, ::3] = np.float16(-1.0e-6)         # a mix of subnormals
+    refs = refs.copy()
+    refs[1, 3, 7] = np.nan                     # a NaN reference element
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     g = run(cg, h.view(np.uint16), refs, S, N, algo=algo, status=st).cpu().numpy()
     o = orc.drift_scores(h.view(np.uint16), refs, S, N)
@@ -214,3 +216,4 @@ def test_drift_infinite_and_extreme_live_values(cg, orc, algo):
     assert_scores_close(g, o, what=f"algo {algo}")
     for n in (1, 2, 3):
         assert np.isinf(g[0, n, 0]) and np.isinf(g[1, n, 0]) and np.isnan(g[2, n, 0])
+    assert np.isnan(g[0, 3, 1]) and np.isnan(g[2, 3, 1]) and np.isfinite(g[1, 3, 1])
