@@ -152,7 +152,7 @@ def test_pooled_nan_flag(cg, orc):
     assert np.array_equal(g["u2"].cpu().numpy(), o["u2"])
 
 
-@pytest.mark.parametrize("C,N,S", [(2, 5, 8), (400, 8, 16), (2, 3, 40), (320, 33, 4)],
+@pytest.mark.parametrize("C,N,S", [(2, 5, 8), (1300, 8, 16), (2, 3, 40), (1300, 33, 4)],
                          ids=["block", "lane_config", "wide", "lane_config_S4"])
 def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
     """A NaN score on a stage the labels exclude (-1) is not part of any pair:
@@ -176,7 +176,7 @@ def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
     assert np.array_equal(gp["auroc"].cpu().numpy().view(np.uint64), op["auroc"].view(np.uint64))
 
 
-@pytest.mark.parametrize("C,N,S", [(3, 40, 8), (400, 8, 16), (2, 6, 40)],
+@pytest.mark.parametrize("C,N,S", [(3, 40, 8), (1300, 8, 16), (2, 6, 40)],
                          ids=["block", "lane_config", "wide"])
 def test_auroc_infinities_and_signed_zero(cg, orc, C, N, S):
     """Scores of +inf (a drift score of an infinite activation), -inf, +0 and
