@@ -379,8 +379,8 @@ def run_ours(args, ranks: Ranks):
     outs_c = {k: torch.empty((1, N), dtype=torch.int64, device=dev) for k in ("u2", "gt", "eq")}
     auroc = torch.empty((2,), dtype=torch.float64, device=dev)
     # drift (pipeline kernel + finalize), control labels, and two AUROC calls
-    # of one configuration (canary-parallel counts + per-configuration combine)
-    launches_per_step = 2 + 1 + 2 * 2
+    # of one configuration
+    launches_per_step = 2 + 1 + 2 * auroc_launches(N, S)
 
     algo = {"auto": None, "stream": cg.DRIFT_STREAM, "bulk": cg.DRIFT_BULK,
             "bulk2": cg.DRIFT_BULK_2CTA}[args.drift_algo]
@@ -847,12 +847,18 @@ def run_study(args, ranks: Ranks):
     print(json.dumps(line), flush=True)
 
 
+def auroc_launches(N, S) -> int:
+    """Launches of one cg_auroc call on a single configuration: one block
+    ranks and combines it (S <= 32, N <= 1024), else canary-parallel counts
+    and a per-configuration combine."""
+    return 1 if S <= 32 and N <= 1024 else 2
+
+
 def launches_per_config(cfg) -> int:
     """Kernel launches of one study configuration: generator (2 when every
     stage's live values follow element by element, else 4; 2 + 3 per stage
     when propagating), drift scores (2), control labels (1), three per-canary
-    AUROC calls and the control's (2 launches each for a single
-    configuration), pooled AUROC (1)."""
+    AUROC calls and the control's, pooled AUROC (1)."""
     if cfg.get("gain", 0.0):
         gen = 2 + 3 * cfg["n_shards"]
     else:
@@ -860,7 +866,7 @@ def launches_per_config(cfg) -> int:
         needs_stats = ((n_mal < cfg["n_shards"] and cfg["noise"] == SI.NOISE_PAPER) or
                        (n_mal > 0 and cfg["tamper"] == SI.TAMPER_ADDITIVE))
         gen = 4 if needs_stats else 2
-    return gen + 2 + 1 + 4 * 2 + 1
+    return gen + 2 + 1 + 4 * auroc_launches(cfg["n_canaries"], cfg["n_shards"]) + 1
 
 
 def study_oracle_baseline(cfgs, seconds):
