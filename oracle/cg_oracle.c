@@ -526,6 +526,46 @@ int or_generate_pipeline(const or_desc *D, uint16_t *acts, float *refs,
   return err;
 }
 
+/* Segments first .. first + count - 1 of the pipeline (segment q = s*N+n),  */
+/* written one after another to acts/refs [count][T*d]: the same values as   */
+/* the matching slice of or_generate_pipeline, for pipelines too large to    */
+/* hold whole on the host (one stage at a time).  coef [count] (may be NULL) */
+/* receives each segment's scalar as or_generate_segment returns it.         */
+int or_generate_segments(const or_desc *D, uint64_t first, uint64_t count,
+                         uint16_t *acts, float *refs, double *coef,
+                         int n_threads) {
+  int st = check_desc(D);
+  if (st) return st;
+  const uint64_t n_seg = (uint64_t)D->n_shards * D->n_canaries;
+  if (first > n_seg || count > n_seg - first) return OR_BAD_ARG;
+  or_tables t;
+  st = build_tables(D, &t);
+  if (st) return st;
+  const uint32_t N = D->n_canaries;
+  const uint64_t L = (uint64_t)D->tokens * D->hidden;
+  int err = OR_OK;
+#ifdef _OPENMP
+  if (n_threads > 0) omp_set_num_threads(n_threads);
+#pragma omp parallel for schedule(dynamic, 1)
+#endif
+  for (int64_t i = 0; i < (int64_t)count; ++i) {
+    const uint64_t q = first + (uint64_t)i;
+    uint32_t s = (uint32_t)(q / N), n = (uint32_t)(q % N);
+    size_t off = (size_t)i * L;
+    int e = segment(D, &t, s, n, refs ? refs + off : NULL, NULL,
+                    acts ? acts + off : NULL, coef ? coef + i : NULL);
+    if (e) {
+#ifdef _OPENMP
+#pragma omp critical
+#endif
+      err = e;
+    }
+  }
+  free_tables(&t);
+  (void)n_threads;
+  return err;
+}
+
 /* Propagating pipeline (Eq. 2's recursion h_i = f_i(h_{i-1}) + delta_i     */
 /* with the block's response to its input linearised as                     */
 /*     f_i(h_{i-1}) = a_i + gain * (h_{i-1} - a_{i-1}),                     */

@@ -115,6 +115,9 @@ def lib():
             L.or_generate_propagating.argtypes = [P(_Desc), dbl, P(ctypes.c_uint16), P(ctypes.c_float),
                                                   ctypes.c_int]
             L.or_generate_propagating.restype = i32
+            L.or_generate_segments.argtypes = [P(_Desc), u64, u64, P(ctypes.c_uint16),
+                                               P(ctypes.c_float), P(dbl), ctypes.c_int]
+            L.or_generate_segments.restype = i32
         return _lib
 
 
@@ -241,6 +244,36 @@ def generate_pipeline(desc, n_threads=0):
                                       _p(refs, ctypes.c_float), _p(labels, ctypes.c_int8),
                                       int(n_threads)))
     return acts, refs, labels
+
+
+def generate_segments(desc, first, count, n_threads=0):
+    """Segments first .. first + count - 1 (segment q = s * N + n): acts
+    (uint16 binary16 bits) and refs (float32), both [count][T*d], equal to
+    that slice of generate_pipeline, and each segment's scalar coef [count]
+    (sigma_s mu under Eq. 2 noise, eps ||a|| / ||g|| under the Gaussian
+    tamper, else 0; as generate_segment returns it)."""
+    L = desc.tokens * desc.hidden
+    acts = np.zeros((count, L), dtype=np.uint16)
+    refs = np.zeros((count, L), dtype=np.float32)
+    coef = np.zeros(count, dtype=np.float64)
+    _check(lib().or_generate_segments(ctypes.byref(desc), first, count,
+                                      _p(acts, ctypes.c_uint16), _p(refs, ctypes.c_float),
+                                      _p(coef, ctypes.c_double), int(n_threads)))
+    return acts, refs, coef
+
+
+def generate_stage(desc, s, n_threads=0):
+    """Every canary of stage s: acts uint16 and refs float32 [N][T*d], coef [N]."""
+    N = desc.n_canaries
+    return generate_segments(desc, s * N, N, n_threads)
+
+
+def generate_coefs(desc, n_threads=0):
+    """The whole pipeline as generate_segments gives it: acts, refs
+    [S][N][T*d] and coef [S][N]."""
+    S, N, L = desc.n_shards, desc.n_canaries, desc.tokens * desc.hidden
+    acts, refs, coef = generate_segments(desc, 0, S * N, n_threads)
+    return acts.reshape(S, N, L), refs.reshape(S, N, L), coef.reshape(S, N)
 
 
 def generate_propagating(desc, gain, n_threads=0):

@@ -176,3 +176,28 @@ def test_tiny_pipeline_detects(orc):
     # the malicious stage's mismatch tracks eps, the benign floor tracks sigma (Sec. 3.4)
     assert np.allclose(sc[0][:, 1], 0.05, rtol=0.02)
     assert sc[0][:, [0, 2, 3]].max() < 3e-3
+
+
+def test_segment_ranges_equal_pipeline_slices(orc):
+    """generate_segments / generate_stage return exactly the matching slice of
+    the whole pipeline (the full-size GPU tests compare one stage at a time),
+    and each segment's scalar as generate_segment gives it."""
+    from oracle.oracle import OracleError
+    for tamper, noise in [(SI.TAMPER_ADDITIVE, SI.NOISE_PAPER), (SI.TAMPER_SCALE, SI.NOISE_MULT)]:
+        cfg = SI.shrink(SI.SEVEN_B, n_shards=3, hidden=24, n_canaries=5, tokens=3, malicious=(1,),
+                        tamper=tamper, tamper_param=0.05 if tamper == SI.TAMPER_ADDITIVE else 1.1,
+                        noise=noise)
+        D = orc.desc_from_dict(cfg)
+        acts, refs, _ = orc.generate_pipeline(D)
+        for s in range(3):
+            a, r, c = orc.generate_stage(D, s)
+            assert np.array_equal(a, acts[s]) and np.array_equal(r, refs[s])
+            for n in range(5):
+                assert c[n] == orc.generate_segment(D, s, n)[3]
+        a, r, c = orc.generate_segments(D, 4, 7)      # crosses the stage 0 / stage 1 boundary
+        assert np.array_equal(a, acts.reshape(15, -1)[4:11])
+        assert np.array_equal(r, refs.reshape(15, -1)[4:11])
+        a, r, c = orc.generate_coefs(D)
+        assert np.array_equal(a, acts) and np.array_equal(r, refs) and c.shape == (3, 5)
+        with pytest.raises(OracleError):
+            orc.generate_segments(D, 10, 6)
