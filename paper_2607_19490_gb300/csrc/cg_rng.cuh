@@ -110,29 +110,6 @@ __device__ __forceinline__ float2 box_muller(uint32_t x0, uint32_t x1) {
   return make_float2(r * cs.x, r * cs.y);
 }
 
-// Box-Muller for the draws that only perturb a live value (benign noise, the
-// Gaussian tamper's direction): the radius takes the special-function
-// log2 (__logf) instead of logf.  Such a normal enters an fp16 live value
-// scaled by sigma_s mu or eps ||a|| / ||g||, at most about 0.1, so the
-// approximation moves the value by far less than its fp16 rounding step.
-// -2 ln u1 is clamped at 0: for u1 just below 1 the approximate log may come
-// out slightly positive.  The references keep box_muller.
-__device__ __forceinline__ float2 box_muller_perturb(uint32_t x0, uint32_t x1) {
-  const float u1 = (float)((x0 >> 8) + 1u) * 0x1p-24f;
-  const float r = sqrt_approx(fmaxf(-2.0f * __logf(u1), 0.0f));
-  const float2 cs = sincos_2pi_u24(x1 >> 8);
-  return make_float2(r * cs.x, r * cs.y);
-}
-
-// The four perturbation normals of one Philox block (box_muller_perturb).
-__device__ __forceinline__ float4 perturb_normals4_rk(const PhiloxRoundKeys &rk, uint32_t q,
-                                                      uint32_t c1, uint32_t c2, uint32_t c3) {
-  const uint4 w = philox4x32_10_rk(make_uint4(q, c1, c2, c3), rk);
-  const float2 a = box_muller_perturb(w.x, w.y);
-  const float2 b = box_muller_perturb(w.z, w.w);
-  return make_float4(a.x, a.y, b.x, b.y);
-}
-
 // The four normals of one Philox block from precomputed round keys (counter
 // word 3 = c3: 0 for every live draw, the replica index for an independent
 // benign recompute).

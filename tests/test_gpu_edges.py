@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 
 import seeded_inputs as SI
-from tests._cmp import assert_normals_close, half_ulp_distance
+from tests._cmp import assert_live_close, assert_normals_close, half_ulp_distance
 
 pytestmark = pytest.mark.gpu
 
@@ -24,11 +24,13 @@ def cg():
 
 def compare(cg, orc, cfg):
     acts, refs, labels = cg.cg_generate_pipeline(cg.PipelineDesc.from_config(cfg))
-    o_acts, o_refs, o_labels = orc.generate_pipeline(orc.desc_from_dict(cfg))
+    D = orc.desc_from_dict(cfg)
+    _, _, o_labels = orc.generate_pipeline(D)
+    o_acts, o_refs, o_coef = orc.generate_coefs(D)
     assert np.array_equal(labels.cpu().numpy(), o_labels)
-    assert_normals_close(refs.cpu().numpy(), o_refs, what="references")
-    d = half_ulp_distance(acts.cpu().numpy().view(np.uint16), o_acts)
-    assert d.max() <= 1
+    g_refs = refs.cpu().numpy()
+    assert_normals_close(g_refs, o_refs, what="references")
+    assert_live_close(acts.cpu().numpy().view(np.uint16), o_acts, g_refs, o_refs, o_coef)
     return acts, refs, labels
 
 

@@ -1,14 +1,15 @@
 """GPU parity of the Philox layer and the pipeline generator against the oracle.
 
 Philox words bit-exact; normals and references within the normal tolerance;
-labels bit-exact; fp16 live values within 1 ulp (tests/_cmp.py).  Inputs are
+labels bit-exact; fp16 live values within the live-value bound of
+tests/_cmp.py (one fp16 step away from cancellations).  Inputs are
 descriptions only, so nothing the oracle sees comes from the CUDA path.
 """
 import numpy as np
 import pytest
 
 import seeded_inputs as SI
-from tests._cmp import assert_normals_close, half_ulp_distance
+from tests._cmp import assert_live_close, assert_normals_close, half_ulp_distance
 
 pytestmark = pytest.mark.gpu
 
@@ -89,29 +90,28 @@ CASES.update({f"factorial_{i}": SI.shrink(c, n_canaries=2, tokens=2)
 
 def compare_pipeline(cg, orc, cfg, acts, refs, labels=None, segments=None):
     """acts/refs: device tensors [S][N][L]; compares the listed (s, n) segments
-    (all when None) against the oracle's generator."""
-    S, N = cfg["n_shards"], cfg["n_canaries"]
+    (all when None) against the oracle's generator.  Returns the largest
+    distance of a live value in fp16 steps."""
     D = orc.desc_from_dict(cfg)
     if segments is None:
-        o_acts, o_refs, o_labels = orc.generate_pipeline(D)
+        o_acts, o_refs, o_coef = orc.generate_coefs(D)
         g_acts = acts.cpu().numpy().view(np.uint16)
         g_refs = refs.cpu().numpy()
         if labels is not None:
+            _, _, o_labels = orc.generate_pipeline(D)
             assert np.array_equal(labels.cpu().numpy(), o_labels)
-        pairs = [(g_acts, g_refs, o_acts, o_refs)]
+        pairs = [(g_acts, g_refs, o_acts, o_refs, o_coef)]
     else:
         pairs = []
         for s, n in segments:
-            o_r, _, o_a, _ = orc.generate_segment(D, s, n)
+            o_r, _, o_a, o_c = orc.generate_segment(D, s, n)
             pairs.append((acts[s, n].cpu().numpy().view(np.uint16), refs[s, n].cpu().numpy(),
-                          o_a, o_r))
+                          o_a, o_r, o_c))
     worst = 0
-    for g_a, g_r, o_a, o_r in pairs:
+    for g_a, g_r, o_a, o_r, o_c in pairs:
         assert_normals_close(g_r, o_r, scale=1.0, what="references")
-        dist = half_ulp_distance(g_a, o_a)
-        worst = max(worst, int(dist.max()))
-        assert dist.max() <= 1, f"live values differ by {dist.max()} fp16 ulp"
-        assert (dist > 0).mean() < 1e-2
+        worst = max(worst, assert_live_close(g_a, o_a, g_r, o_r, o_c))
+        assert (half_ulp_distance(g_a, o_a) > 0).mean() < 1e-2
     return worst
 
 
