@@ -5,8 +5,8 @@ depth (k = 2..12) keep A-hat = 1.000; the frontier holds A-hat = 1.000 down
 to eps = 0.002 at sigma_hw = 0.002 and gives way below it; the noise-floor
 study holds while sigma_hw <= eps and fails once the floor is twice the
 tamper.  The factorial's 324 configurations all separate with relative-L2.
-Smaller copies of sampled configurations are checked against the oracle's
-end-to-end A-hat where it is decisive."""
+Smaller copies of sampled configurations are checked end to end against the
+oracle (generator, drift scores, bit-exact ranking of the GPU's scores)."""
 import json
 import os
 
@@ -34,12 +34,6 @@ def gpu_auroc(cg, cfg, stat=0):
     acts, refs, labels = cg.cg_generate_pipeline(desc)
     sc = cg.cg_drift_scores(acts, refs, cfg["n_shards"], cfg["n_canaries"])
     return cg.cg_auroc(sc[stat][None].contiguous(), labels[None])["auroc"].item()
-
-
-def oracle_auroc(orc, cfg, stat=0):
-    acts, refs, labels = orc.generate_pipeline(orc.desc_from_dict(cfg))
-    sc = orc.drift_scores(acts, refs, cfg["n_shards"], cfg["n_canaries"]).astype(np.float32)
-    return orc.auroc(sc[stat][None], labels[None])["auroc"][0]
 
 
 @pytest.mark.parametrize("study", ["collusion", "position", "depth"])
@@ -91,13 +85,13 @@ def test_factorial_all_separate(cg):
 @pytest.mark.parametrize("study,idx", [("collusion", 9), ("position", 0), ("position", 12),
                                        ("frontier", 15), ("frontier", 18), ("depth", 0),
                                        ("paper_snr", 12), ("paper_snr", 15)])
-def test_matches_oracle_when_decisive(cg, orc, study, idx):
+def test_shrunk_study_configs_match_oracle(cg, orc, study, idx):
+    """Shrunk study configurations end to end: every generated element, every
+    drift score on the GPU's bytes, and u2 / gt / eq / A-hat of the GPU's own
+    scores bit-exact against the oracle's ranking."""
+    from tests._fullpath import check_against_oracle, run_gpu
     cfg = SI.shrink(SI.STUDIES[study]()[idx], n_canaries=16, tokens=8)
-    g, o = gpu_auroc(cg, cfg), oracle_auroc(orc, cfg)
-    if o in (0.0, 1.0):
-        assert g == o
-    else:
-        assert abs(g - o) <= 0.1
+    check_against_oracle(orc, cfg, run_gpu(cg, cfg))
 
 
 @pytest.mark.parametrize("study,idx", [("factorial", 323), ("factorial", 300), ("factorial", 270),
@@ -108,16 +102,17 @@ def test_full_size_configs_sampled_against_oracle(cg, orc, study, idx):
     the generator against the oracle, and neutral bytes planted into sampled
     segments scored in the same launch as the rest of the pipeline."""
     import torch
-    from tests._cmp import assert_normals_close, assert_scores_close, half_ulp_distance
+    from tests._cmp import assert_live_close, assert_normals_close, assert_scores_close
     cfg = SI.STUDIES[study]()[idx]
     S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
     acts, refs, labels = cg.cg_generate_pipeline(cg.PipelineDesc.from_config(cfg))
     D = orc.desc_from_dict(cfg)
     picks = [(0, 0), (cfg["malicious"][0], N - 1), (S // 2, N // 2)]
     for s, n in picks:
-        o_r, _, o_a, _ = orc.generate_segment(D, s, n)
-        assert_normals_close(refs[s, n].cpu().numpy(), o_r, what="references")
-        assert half_ulp_distance(acts[s, n].cpu().numpy().view(np.uint16), o_a).max() <= 1
+        o_r, _, o_a, o_c = orc.generate_segment(D, s, n)
+        g_r = refs[s, n].cpu().numpy()
+        assert_normals_close(g_r, o_r, what="references")
+        assert_live_close(acts[s, n].cpu().numpy().view(np.uint16), o_a, g_r, o_r, o_c)
     planted = {}
     for i, (s, n) in enumerate([(1, 1), (S - 1, 0)]):
         pa, pr = SI.drift_arrays(1, 1, L, seed=900 + i)
