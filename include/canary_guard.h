@@ -28,6 +28,9 @@
  *     maps the word to a cg_status.
  *   - Results are deterministic run to run on one GPU: fixed reduction
  *     order, no floating-point atomics.
+ *   - The library keeps per-device set-up (kernel attributes, occupancy)
+ *     for the life of the process; after cudaDeviceReset, calls on that
+ *     device may fail with CG_ERR_CUDA.
  *   - fp16 tensors are passed as uint16_t binary16 bit patterns.
  *   - Layouts: live activations and references are [S][N][T][d] row-major
  *     (one (stage, canary) segment = T*d contiguous elements); drift
@@ -215,8 +218,13 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * d_scores[stat * stat_stride + n * S + s] (stat_stride >= N * S; pass
  * N * S for a dense [3][N][S] block).  Each element of d_acts and d_refs is
  * read once from HBM.  Sums are accumulated in fp32 per chunk of 16384
- * elements and combined in fp64, so finite element magnitudes must stay
- * below about 1e17 for the squared sums to remain finite.  A NaN element
+ * elements and combined in fp64, so the scores hold their tolerance (rel_l2
+ * within 1e-5 relative) for finite element magnitudes between about 1e-18
+ * and 1e17: above, the squared sums overflow; below about 1e-19 the squares
+ * fall into fp32's subnormal range and lose precision, and below about
+ * 4e-23 they underflow to zero.  A segment whose every squared difference
+ * underflows while some difference is nonzero (all |h - a| < 2^-74.5) gets
+ * rel_l2 and cos_dev NaN, never a wrong finite value.  A NaN element
  * makes rel_l2 and cos_dev NaN (max_abs skips it); an infinite live
  * element (fp16 +-inf, which an untrusted hop may send) makes rel_l2 and
  * max_abs +inf and cos_dev NaN.  d_ws: >= cg_drift_workspace_size bytes,
@@ -251,6 +259,26 @@ cg_status cg_drift_scores_ex(const uint16_t *d_acts, const float *d_refs,
                              int32_t *d_status, int32_t algo, cg_stream_t stream);
 
 /*
+ * cg_drift_scores over a batch of C = n_configs configurations of the same
+ * shape in one launch pair (the factorial and the substudies score many
+ * configurations of equal shape, Sec. 4.4; a launch over several of them
+ * amortises the pipeline's fill and drain).  d_acts fp16 and d_refs fp32
+ * are [C][S][N][seg_len], 16-byte aligned; the scores of configuration c go
+ * to d_scores[stat * stat_stride + c * N * S + n * S + s] (stat_stride >=
+ * C * N * S; pass C * N * S for a dense [3][C][N][S] block, whose per-stat
+ * [C][N][S] slices are cg_auroc's input).  d_ws: >= cg_drift_workspace_size(
+ * C * S, N, seg_len) bytes, 16-byte aligned, scratch.  Kernel choice,
+ * numerics and every other rule are those of cg_drift_scores; C = 1 is
+ * cg_drift_scores itself.
+ */
+cg_status cg_drift_scores_batch(const uint16_t *d_acts, const float *d_refs,
+                                uint32_t n_configs, uint32_t n_shards,
+                                uint32_t n_canaries, uint64_t seg_len,
+                                float *d_scores, uint64_t stat_stride, void *d_ws,
+                                size_t ws_bytes, int32_t *d_status,
+                                cg_stream_t stream);
+
+/*
  * cg_drift_scores with the live activations in pinned host memory: the
  * drift kernel reads h_acts directly over the host-GPU link (one pass, no
  * staging copy in HBM) while the references stay resident in device memory,
@@ -279,10 +307,13 @@ cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs,
  *   Limit: n_shards * n_canaries * ceil(seg_len / CG_NOALLOC_CHUNK_ELEMENTS)
  *   <= CG_NOALLOC_MAX_WORK_ITEMS (e.g. 4096 segments of 2^20 elements);
  *   larger problems return CG_ERR_UNSUPPORTED before any launch.
- *   The array is loaded on every GPU that loads the library and held until
- *   the process exits.  The first call on each device looks up the array's
- *   device address (cudaGetSymbolAddress) with that device current; make
- *   that first call before any stream capture.
+ *   The 4 MiB are held on each device where the library's device code is
+ *   loaded (its first kernel launch or first call of this entry point on
+ *   that device, under CUDA's default lazy module loading) until the
+ *   process exits.  Every call looks up the array's device address
+ *   (cudaGetSymbolAddress) with the current device; the first such lookup on
+ *   a device loads the module there, so make that first call before any
+ *   stream capture.
  *   Every call shares the array: calls that overlap on the GPU (on
  *   different streams or from different host threads) race and corrupt
  *   each other's results; serialise them on one stream.  Nothing in it

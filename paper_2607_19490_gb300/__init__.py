@@ -20,7 +20,8 @@ __all__ = [
     "CgError", "load", "cg_status_string", "cg_abi_version", "PipelineDesc",
     "cg_philox_words", "cg_philox_normals", "cg_box_muller_pairs", "cg_generate_workspace_size",
     "cg_generate_pipeline", "cg_drift_workspace_size", "cg_drift_scores",
-    "cg_drift_scores_ex", "cg_drift_scores_host", "cg_drift_scores_noalloc",
+    "cg_drift_scores_ex", "cg_drift_scores_batch", "cg_drift_scores_host",
+    "cg_drift_scores_noalloc",
     "cg_make_control_labels", "cg_auroc", "cg_read_status", "cg_generate_recompute",
     "cg_random_scores", "cg_auroc_pooled", "cg_generate_propagating", "cg_selftest_bounded_wait",
     "NOISE_MULT", "NOISE_PAPER", "TAMPER_ADDITIVE", "TAMPER_SIGNFLIP_CHANNELS",
@@ -102,6 +103,7 @@ def load() -> ctypes.CDLL:
             "cg_random_scores": ([u64, u32, u32, u32, u32, P, P], ctypes.c_int),
             "cg_drift_scores": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_ex": ([P, P, u32, u32, u64, P, u64, P, sz, P, ctypes.c_int32, P], ctypes.c_int),
+            "cg_drift_scores_batch": ([P, P, u32, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_host": ([P, P, u32, u32, u64, P, u64, P, sz, P, P], ctypes.c_int),
             "cg_drift_scores_noalloc": ([P, P, u32, u32, u64, P, u64, P, P], ctypes.c_int),
             "cg_make_control_labels": ([P, u32, u32, u32, u64, u32, P, P, P], ctypes.c_int),
@@ -139,6 +141,10 @@ def _cuda(t, name, dtypes):
         return
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
+    # the library launches on the current device with the current stream
+    if t.device.index != _torch().cuda.current_device():
+        raise ValueError(f"{name} is on {t.device}, but the current device is "
+                         f"cuda:{_torch().cuda.current_device()}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if t.dtype not in dtypes:
@@ -341,6 +347,39 @@ def cg_drift_scores(acts, refs, n_shards, n_canaries, scores=None, stat_stride=N
                                          _ptr(scores), stat_stride, _ptr(ws), ws.numel(),
                                          _ptr(status), int(algo), _stream(stream)),
                "cg_drift_scores_ex")
+    return scores
+
+
+def cg_drift_scores_batch(acts, refs, n_configs, n_shards, n_canaries, scores=None,
+                          stat_stride=None, ws=None, status=None, stream=None):
+    """Drift scores [3][C][N][S] of C equal-shape configurations, acts fp16 /
+    refs fp32 [C][S][N][L], in one launch pair."""
+    torch = _torch()
+    _cuda(acts, "acts", (torch.float16,))
+    _cuda(refs, "refs", (torch.float32,))
+    n_seg = n_configs * n_shards * n_canaries
+    if acts.numel() != refs.numel() or acts.numel() % n_seg:
+        raise ValueError("acts and refs must both hold C*S*N*L elements")
+    seg_len = acts.numel() // n_seg
+    if scores is None:
+        scores = torch.empty((3, n_configs, n_canaries, n_shards), dtype=torch.float32,
+                             device=acts.device)
+        stat_stride = n_seg
+    if stat_stride is None:
+        stat_stride = n_seg
+    need = cg_drift_workspace_size(n_configs * n_shards, n_canaries, seg_len)
+    if ws is None:
+        ws = torch.empty(need, dtype=torch.uint8, device=acts.device)
+    _cuda(scores, "scores", (torch.float32,))
+    _cuda(ws, "ws", (torch.uint8,))
+    _cuda(status, "status", (torch.int32,))
+    if scores.numel() < 2 * stat_stride + n_seg:
+        raise ValueError("scores must hold 2 * stat_stride + C * N * S floats")
+    if ws.numel() < need:
+        raise ValueError("workspace smaller than cg_drift_workspace_size(C * S, N, L)")
+    _check(load().cg_drift_scores_batch(_ptr(acts), _ptr(refs), n_configs, n_shards, n_canaries,
+                                        seg_len, _ptr(scores), stat_stride, _ptr(ws), ws.numel(),
+                                        _ptr(status), _stream(stream)), "cg_drift_scores_batch")
     return scores
 
 

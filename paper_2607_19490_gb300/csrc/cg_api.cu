@@ -138,6 +138,36 @@ cg::GenParams make_params(const cg_pipeline_desc &d, const cg::GenLayout &lay) {
   return p;
 }
 
+// Argument checks and kernel choice shared by the drift entry points: C
+// configurations of S stages x N canaries, [C][S][N][seg_len].
+cg_status drift_scores_checked(const uint16_t *d_acts, const float *d_refs, uint32_t n_configs,
+                               uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
+                               float *d_scores, uint64_t stat_stride, void *d_ws, size_t ws_bytes,
+                               int32_t *d_status, int32_t algo, cg_stream_t stream) {
+  if (!d_acts || !d_refs || !d_scores || n_configs == 0 || n_shards == 0 || n_canaries == 0 ||
+      seg_len == 0)
+    return CG_ERR_INVALID_ARG;
+  if (algo < CG_DRIFT_AUTO || algo > CG_DRIFT_BULK_2CTA) return CG_ERR_INVALID_ARG;
+  const uint64_t n_seg = (uint64_t)n_configs * n_shards * n_canaries;
+  if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
+  if (stat_stride < n_seg) return CG_ERR_INVALID_ARG;
+  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || !aligned(d_scores, 4) ||
+      (d_status && !aligned(d_status, 4)))
+    return CG_ERR_ALIGNMENT;
+  if (!d_ws || ws_bytes < cg::drift_ws_bytes(n_seg, seg_len)) return CG_ERR_WORKSPACE;
+  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
+  // The bulk-copy pipelines take device memory only (8-element aligned
+  // segments); anything else streams through registers.
+  const bool bulk_ok = cg::drift_bulk_eligible(d_acts, d_refs, seg_len) &&
+                       is_device_memory(d_acts) && is_device_memory(d_refs);
+  if ((algo == CG_DRIFT_BULK || algo == CG_DRIFT_BULK_2CTA) && !bulk_ok)
+    return CG_ERR_UNSUPPORTED;
+  if (algo == CG_DRIFT_AUTO) algo = bulk_ok ? CG_DRIFT_BULK : CG_DRIFT_STREAM;
+  return from_cuda(cg::launch_drift_algo(d_acts, d_refs, n_configs, n_shards, n_canaries,
+                                         seg_len, d_scores, stat_stride, d_ws, d_status, algo,
+                                         (cudaStream_t)stream));
+}
+
 }  // namespace
 
 extern "C" {
@@ -283,27 +313,17 @@ cg_status cg_drift_scores_ex(const uint16_t *d_acts, const float *d_refs, uint32
                              uint64_t stat_stride, void *d_ws, size_t ws_bytes, int32_t *d_status,
                              int32_t algo, cg_stream_t stream) {
   CG_TRACE("cg_drift_scores_ex");
-  if (!d_acts || !d_refs || !d_scores || n_shards == 0 || n_canaries == 0 || seg_len == 0)
-    return CG_ERR_INVALID_ARG;
-  if (algo < CG_DRIFT_AUTO || algo > CG_DRIFT_BULK_2CTA) return CG_ERR_INVALID_ARG;
-  const uint64_t n_seg = (uint64_t)n_shards * n_canaries;
-  if (stat_stride < n_seg) return CG_ERR_INVALID_ARG;
-  if (seg_len > (1ull << 40) || n_seg > (1ull << 31)) return CG_ERR_UNSUPPORTED;
-  if (!aligned(d_acts, 16) || !aligned(d_refs, 16) || !aligned(d_scores, 4) ||
-      (d_status && !aligned(d_status, 4)))
-    return CG_ERR_ALIGNMENT;
-  if (!d_ws || ws_bytes < cg::drift_ws_bytes(n_seg, seg_len)) return CG_ERR_WORKSPACE;
-  if (!aligned(d_ws, 16)) return CG_ERR_ALIGNMENT;
-  // The bulk-copy pipelines take device memory only (8-element aligned
-  // segments); anything else streams through registers.
-  const bool bulk_ok = cg::drift_bulk_eligible(d_acts, d_refs, seg_len) &&
-                       is_device_memory(d_acts) && is_device_memory(d_refs);
-  if ((algo == CG_DRIFT_BULK || algo == CG_DRIFT_BULK_2CTA) && !bulk_ok)
-    return CG_ERR_UNSUPPORTED;
-  if (algo == CG_DRIFT_AUTO) algo = bulk_ok ? CG_DRIFT_BULK : CG_DRIFT_STREAM;
-  return from_cuda(cg::launch_drift_algo(d_acts, d_refs, n_shards, n_canaries, seg_len, d_scores,
-                                         stat_stride, d_ws, d_status, algo,
-                                         (cudaStream_t)stream));
+  return drift_scores_checked(d_acts, d_refs, 1, n_shards, n_canaries, seg_len, d_scores,
+                              stat_stride, d_ws, ws_bytes, d_status, algo, stream);
+}
+
+cg_status cg_drift_scores_batch(const uint16_t *d_acts, const float *d_refs, uint32_t n_configs,
+                                uint32_t n_shards, uint32_t n_canaries, uint64_t seg_len,
+                                float *d_scores, uint64_t stat_stride, void *d_ws,
+                                size_t ws_bytes, int32_t *d_status, cg_stream_t stream) {
+  CG_TRACE("cg_drift_scores_batch");
+  return drift_scores_checked(d_acts, d_refs, n_configs, n_shards, n_canaries, seg_len, d_scores,
+                              stat_stride, d_ws, ws_bytes, d_status, CG_DRIFT_AUTO, stream);
 }
 
 cg_status cg_drift_scores_host(const uint16_t *h_acts, const float *d_refs, uint32_t n_shards,

@@ -24,12 +24,26 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // ---------------------------------------------------------------- drift
 // A work item is a chunk of at most kDriftChunk elements of one segment.
+// A segment has ceil(L / kDriftChunk) items (this count sizes the
+// workspace); they share the segment evenly in whole multiples of
+// kDriftItemGranule elements, the bulk pipeline's stage, so that no item is
+// a short remainder (L = 36,864: three items of 12,288, not 16,384 + 16,384
+// + 4,096).  Only the last item of a segment may be shorter.
 constexpr uint32_t kDriftChunk = 16384;
+constexpr uint32_t kDriftItemGranule = 4096;
 constexpr int kDriftThreads = 256;
 constexpr size_t kDriftHeader = 256;   // reserved bytes at the start of the workspace
 
 inline uint64_t drift_chunks_per_seg(uint64_t seg_len) {
   return (seg_len + kDriftChunk - 1) / kDriftChunk;
+}
+// Elements per item: ceil(L / items) rounded up to the granule.  It is at
+// most kDriftChunk (a multiple of the granule), and items - 1 of them cover
+// less than L, so the last item is never empty.
+inline uint64_t drift_item_len(uint64_t seg_len) {
+  const uint64_t items = drift_chunks_per_seg(seg_len);
+  const uint64_t even = (seg_len + items - 1) / items;
+  return (even + kDriftItemGranule - 1) / kDriftItemGranule * kDriftItemGranule;
 }
 inline size_t drift_ws_bytes(uint64_t n_segments, uint64_t seg_len) {
   return kDriftHeader + align_up((size_t)(n_segments * drift_chunks_per_seg(seg_len)) * 16, 256);
@@ -38,9 +52,11 @@ inline size_t drift_ws_bytes(uint64_t n_segments, uint64_t seg_len) {
 
 cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream);
 bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_len);
-cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
-                              uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
-                              int32_t *status, int algo, cudaStream_t stream);
+// C configurations of S stages x N canaries, [C][S][N][seg_len]; scores of
+// configuration c, stage s, canary n at stat * stat_stride + c N S + n S + s.
+cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t C, uint32_t S,
+                              uint32_t N, uint64_t seg_len, float *scores, uint64_t stat_stride,
+                              void *ws, int32_t *status, int algo, cudaStream_t stream);
 
 // Work-item capacity of the fixed scratch array used by cg_drift_scores_noalloc.
 constexpr uint64_t kNoallocDriftItems = 262144;

@@ -3,8 +3,9 @@
 // verifier: every fp16 live element and every fp32 reference element is
 // read exactly once (6 bytes per element).
 //
-// Pass 1 cuts the [S][N][L] element space into work items of at most
-// kDriftChunk elements, never crossing a segment, and writes one float4 of
+// Pass 1 cuts the [C][S][N][L] element space into work items of at most
+// kDriftChunk elements (drift_item_len: even shares of a segment in whole
+// 4,096-element stages), never crossing a segment, and writes one float4 of
 // fp32 sums per item:
 //     D = sum (h - a)^2,   E = sum (h - a)(h + a) = sum h^2 - a^2,
 //     A = sum a^2,         M = max |h - a|
@@ -86,7 +87,7 @@ constexpr int kUnroll = 4;
 
 __global__ void __launch_bounds__(kDriftThreads)
 drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ refs,
-                     uint64_t L, uint64_t chunks_per_seg, uint64_t n_items,
+                     uint64_t L, uint64_t chunks_per_seg, uint64_t item_len, uint64_t n_items,
                      float4 *__restrict__ partials) {
   __shared__ Acc warp_acc[kDriftThreads / 32];
   const int tid = threadIdx.x;
@@ -94,8 +95,8 @@ drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict_
     const uint64_t seg = item / chunks_per_seg;
     const uint64_t ch = item - seg * chunks_per_seg;
     const uint64_t seg0 = seg * L;
-    const uint64_t g0 = seg0 + ch * kDriftChunk;
-    const uint64_t g1 = min(g0 + (uint64_t)kDriftChunk, seg0 + L);
+    const uint64_t g0 = seg0 + ch * item_len;
+    const uint64_t g1 = min(g0 + item_len, seg0 + L);
     Acc s = {0.f, 0.f, 0.f, 0.f};
 
     uint64_t v0 = (g0 + 7) & ~(uint64_t)7;
@@ -162,15 +163,18 @@ drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict_
 //             (D - (sqrt H - sqrt A)^2) / (2 sqrt(H A)) without cancelling
 //             two near-equal norms.
 // One warp per segment: lane l adds the items l, l + 32, ... in order in
-// fp64, then a fixed shuffle tree combines the lanes.
+// fp64, then a fixed shuffle tree combines the lanes.  Segment
+// q = (c S + s) N + n of C configurations writes its scores at
+// stat * stat_stride + c N S + n S + s.
 constexpr int kFinThreads = 256;
 
 __global__ void __launch_bounds__(kFinThreads)
-drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg, uint32_t S,
-                      uint32_t N, float *__restrict__ scores, uint64_t stat_stride) {
+drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg, uint32_t C,
+                      uint32_t S, uint32_t N, float *__restrict__ scores, uint64_t stat_stride) {
   const uint64_t seg = ((uint64_t)blockIdx.x * kFinThreads + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
-  if (seg >= (uint64_t)S * N) return;          // whole warps leave together
+  const uint64_t per_config = (uint64_t)S * N;
+  if (seg >= (uint64_t)C * per_config) return;   // whole warps leave together
   double D = 0.0, E = 0.0, A = 0.0;
   float M = 0.f;
   const float4 *p = partials + seg * chunks_per_seg;
@@ -193,7 +197,12 @@ drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_s
   // FP64 pipe is narrow, and fp32 sqrt/div of the rounded sums is accurate
   // to a few 1e-7 relative, far inside the drift tolerances).
   float rel, cosd;
-  if (isnan(D) || isnan(A)) {
+  // D >= M^2 holds for the exact sums, so D == 0 with M > 0 means every
+  // squared difference underflowed fp32 (all |h - a| below about 2^-74.5):
+  // the segment lies below the range the fp32 sums resolve, and its scores
+  // are NaN rather than a wrong number.
+  const bool underflow = (M > 0.f) && (D == 0.0);
+  if (isnan(D) || isnan(A) || underflow) {
     rel = NAN;
   } else if (A > 0.0) {
     rel = sqrtf((float)D / (float)A);
@@ -201,7 +210,7 @@ drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_s
     rel = (D == 0.0) ? 0.f : INFINITY;
   }
   const double H = A + E;
-  if (isnan(D) || isnan(E) || isnan(A)) {
+  if (isnan(D) || isnan(E) || isnan(A) || underflow) {
     cosd = NAN;
   } else if (H > 0.0 && A > 0.0 && (isinf(D) || isinf(E))) {
     cosd = NAN;                                  // an infinite live element: h / |h| is inf / inf
@@ -213,19 +222,21 @@ drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_s
   } else {
     cosd = 0.f;
   }
-  const uint32_t s = (uint32_t)(seg / N), n = (uint32_t)(seg % N);
-  const uint64_t o = (uint64_t)n * S + s;
+  const uint64_t c = seg / per_config, r = seg - c * per_config;
+  const uint32_t s = (uint32_t)(r / N), n = (uint32_t)(r % N);
+  const uint64_t o = c * per_config + (uint64_t)n * S + s;
   scores[o] = rel;
   scores[stat_stride + o] = M;
   scores[2 * stat_stride + o] = cosd;
 }
 
-static cudaError_t launch_finalize(const float4 *partials, uint64_t cps, uint32_t S, uint32_t N,
-                                   float *scores, uint64_t stat_stride, cudaStream_t stream) {
-  const uint64_t n_seg = (uint64_t)S * N;
+static cudaError_t launch_finalize(const float4 *partials, uint64_t cps, uint32_t C, uint32_t S,
+                                   uint32_t N, float *scores, uint64_t stat_stride,
+                                   cudaStream_t stream) {
+  const uint64_t n_seg = (uint64_t)C * S * N;
   const uint64_t blocks = (n_seg * 32 + kFinThreads - 1) / kFinThreads;
-  drift_finalize_kernel<<<(unsigned)blocks, kFinThreads, 0, stream>>>(partials, cps, S, N, scores,
-                                                                      stat_stride);
+  drift_finalize_kernel<<<(unsigned)blocks, kFinThreads, 0, stream>>>(partials, cps, C, S, N,
+                                                                      scores, stat_stride);
   return cudaGetLastError();
 }
 
@@ -319,8 +330,8 @@ struct BulkSmem {
 template <int NS>
 __global__ void __launch_bounds__(kBulkThreads)
 drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ refs, uint64_t L,
-                  uint64_t chunks_per_seg, uint64_t n_items, float4 *__restrict__ partials,
-                  int32_t *status) {
+                  uint64_t chunks_per_seg, uint64_t item_len, uint64_t n_items,
+                  float4 *__restrict__ partials, int32_t *status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   BulkSmem<NS> &sm = *reinterpret_cast<BulkSmem<NS> *>(smem_raw);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -345,8 +356,8 @@ drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ r
     for (uint64_t item = blockIdx.x; item < n_items && ok; item += gridDim.x) {
       const uint64_t seg = item / chunks_per_seg;
       const uint64_t ch = item - seg * chunks_per_seg;
-      const uint64_t g0 = seg * L + ch * kDriftChunk;
-      const uint64_t len = min((uint64_t)kDriftChunk, L - ch * kDriftChunk);
+      const uint64_t g0 = seg * L + ch * item_len;
+      const uint64_t len = min(item_len, L - ch * item_len);
       for (uint64_t off = 0; off < len; off += kBulkStageElems, ++stage) {
         const uint32_t n = (uint32_t)min((uint64_t)kBulkStageElems, len - off);
         const int slot = (int)(stage % NS);
@@ -382,7 +393,7 @@ drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ r
   uint32_t stage = 0, local_item = 0;
   for (uint64_t item = blockIdx.x; item < n_items; item += gridDim.x, ++local_item) {
     const uint64_t ch = item % chunks_per_seg;
-    const uint64_t len = min((uint64_t)kDriftChunk, L - ch * kDriftChunk);
+    const uint64_t len = min(item_len, L - ch * item_len);
     Acc s = {0.f, 0.f, 0.f, 0.f};
     for (uint64_t off = 0; off < len; off += kBulkStageElems, ++stage) {
       const uint32_t n = (uint32_t)min((uint64_t)kBulkStageElems, len - off);
@@ -456,8 +467,9 @@ drift_bulk_kernel(const uint16_t *__restrict__ acts, const float *__restrict__ r
 
 template <int NS>
 static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t seg_len,
-                               uint64_t cps, uint64_t n_items, float4 *partials, int32_t *status,
-                               int sm_count, cudaStream_t stream) {
+                               uint64_t cps, uint64_t item_len, uint64_t n_items,
+                               float4 *partials, int32_t *status, int sm_count,
+                               cudaStream_t stream) {
   const size_t smem = sizeof(BulkSmem<NS>);
   // shared-memory opt-in and occupancy, once per device
   static std::mutex mu;
@@ -484,8 +496,8 @@ static cudaError_t launch_bulk(const uint16_t *acts, const float *refs, uint64_t
   }
   uint64_t grid = (uint64_t)sm_count * (uint64_t)per_sm;
   if (grid > n_items) grid = n_items;
-  drift_bulk_kernel<NS><<<(unsigned)grid, kBulkThreads, smem, stream>>>(acts, refs, seg_len, cps,
-                                                                        n_items, partials, status);
+  drift_bulk_kernel<NS><<<(unsigned)grid, kBulkThreads, smem, stream>>>(
+      acts, refs, seg_len, cps, item_len, n_items, partials, status);
   return cudaGetLastError();
 }
 
@@ -509,30 +521,33 @@ bool drift_bulk_eligible(const uint16_t *acts, const float *refs, uint64_t seg_l
   return (seg_len % 8) == 0 && ((uintptr_t)acts % 16) == 0 && ((uintptr_t)refs % 16) == 0;
 }
 
-cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t S, uint32_t N,
-                              uint64_t seg_len, float *scores, uint64_t stat_stride, void *ws,
-                              int32_t *status, int algo, cudaStream_t stream) {
+cudaError_t launch_drift_algo(const uint16_t *acts, const float *refs, uint32_t C, uint32_t S,
+                              uint32_t N, uint64_t seg_len, float *scores, uint64_t stat_stride,
+                              void *ws, int32_t *status, int algo, cudaStream_t stream) {
   DeviceInfo info;
   if (!device_info(&info)) return cudaGetLastError();
-  const uint64_t n_seg = (uint64_t)S * N;
+  const uint64_t n_seg = (uint64_t)C * S * N;
   const uint64_t cps = drift_chunks_per_seg(seg_len);
+  const uint64_t item_len = drift_item_len(seg_len);
   const uint64_t n_items = n_seg * cps;
   float4 *partials = reinterpret_cast<float4 *>(static_cast<char *>(ws) + kDriftHeader);
   cudaError_t err;
   if (algo == CG_DRIFT_BULK) {
-    err = launch_bulk<6>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
+    err = launch_bulk<6>(acts, refs, seg_len, cps, item_len, n_items, partials, status,
+                         info.sm_count, stream);
   } else if (algo == CG_DRIFT_BULK_2CTA) {
-    err = launch_bulk<4>(acts, refs, seg_len, cps, n_items, partials, status, info.sm_count, stream);
+    err = launch_bulk<4>(acts, refs, seg_len, cps, item_len, n_items, partials, status,
+                         info.sm_count, stream);
   } else {
     uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
     if (grid > n_items) grid = n_items;
     if (grid < 1) grid = 1;
     drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
-                                                                       n_items, partials);
+                                                                       item_len, n_items, partials);
     err = cudaGetLastError();
   }
   if (err != cudaSuccess) return err;
-  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
+  return launch_finalize(partials, cps, C, S, N, scores, stat_stride, stream);
 }
 
 cudaError_t launch_bounded_wait_probe(uint32_t limit_us, int32_t *status, cudaStream_t stream) {
@@ -553,32 +568,25 @@ int drift_occupancy() {
 // ----------------------------------------------------------------- no-alloc variant
 // Scratch for cg_drift_scores_noalloc: the per-item partial sums live in a
 // fixed device array owned by the library instead of a caller workspace.
-// 262,144 float4 items = 4 MiB, held on every GPU that loads the library
-// until the process exits.  All calls share it, so calls that overlap on the
-// GPU (different streams, or other host threads) race on it.
+// 262,144 float4 items = 4 MiB on each device where this module is loaded
+// (its first kernel launch or first no-alloc call there), until the process
+// exits.  All calls share it, so calls that overlap on the GPU (different
+// streams, or other host threads) race on it.
 static __device__ __align__(256) float4 g_drift_scratch[cg::kNoallocDriftItems];
 
 namespace cg {
-namespace {
-std::mutex g_scratch_mu;
-float4 *g_scratch_ptr[64] = {};
-}  // namespace
 
-// Device address of g_drift_scratch on the current device, looked up once
-// per device (cudaGetSymbolAddress; the host-side symbol is only a stand-in).
+// Device address of g_drift_scratch on the current device.  The host-side
+// symbol is only a stand-in, so the address is looked up with
+// cudaGetSymbolAddress.  It is looked up on every call: the lookup is cheap
+// next to a launch, and an address kept from an earlier call would point at
+// freed memory after the device's context is reset and the module reloaded.
+// The first lookup on a device loads the module there.
 static cudaError_t noalloc_scratch(float4 **out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void *p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_drift_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
-    void *p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_drift_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_ptr[dev] = static_cast<float4 *>(p);
-  }
-  *out = g_scratch_ptr[dev];
+  *out = static_cast<float4 *>(p);
   return cudaSuccess;
 }
 
@@ -596,11 +604,11 @@ cudaError_t launch_drift_noalloc(const uint16_t *acts, const float *refs, uint32
   uint64_t grid = (uint64_t)info.sm_count * (uint64_t)info.drift_blocks_per_sm;
   if (grid > n_items) grid = n_items;
   if (grid < 1) grid = 1;
-  drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(acts, refs, seg_len, cps,
-                                                                     n_items, partials);
+  drift_partial_kernel<<<(unsigned)grid, kDriftThreads, 0, stream>>>(
+      acts, refs, seg_len, cps, drift_item_len(seg_len), n_items, partials);
   err = cudaGetLastError();
   if (err != cudaSuccess) return err;
-  return launch_finalize(partials, cps, S, N, scores, stat_stride, stream);
+  return launch_finalize(partials, cps, 1, S, N, scores, stat_stride, stream);
 }
 
 }  // namespace cg

@@ -153,7 +153,8 @@ def test_drift_host_rejects_pageable(cg):
 
 @pytest.mark.parametrize("algo", [1, 2, 3])
 @pytest.mark.parametrize("S,N,L", [(2, 3, 8), (4, 4, 104), (2, 2, 16384), (3, 5, 40000),
-                                   (1, 2, 65536 + 8), (5, 7, 4096), (4, 16, 8192), (2, 3, 4096 * 3 + 8)])
+                                   (1, 2, 65536 + 8), (5, 7, 4096), (4, 16, 8192), (2, 3, 4096 * 3 + 8),
+                                   (3, 4, 36864), (2, 3, 16392), (2, 2, 4 * 16384 + 8)])
 def test_drift_kernels_match_oracle(cg, orc, algo, S, N, L):
     """The register-streaming kernel and both TMA bulk-copy pipelines against
     the oracle; the bulk pipelines' bounded waits never give up."""
@@ -217,3 +218,61 @@ def test_drift_infinite_and_extreme_live_values(cg, orc, algo):
     for n in (1, 2, 3):
         assert np.isinf(g[0, n, 0]) and np.isinf(g[1, n, 0]) and np.isnan(g[2, n, 0])
     assert np.isnan(g[0, 3, 1]) and np.isnan(g[2, 3, 1]) and np.isfinite(g[1, 3, 1])
+
+
+@pytest.mark.parametrize("C,S,N,L", [(5, 3, 4, 36864), (3, 2, 5, 16385), (7, 4, 3, 8),
+                                     (2, 12, 10, 4096 * 3 + 8), (4, 2, 3, 1)])
+def test_drift_batch_matches_oracle(cg, orc, C, S, N, L):
+    """cg_drift_scores_batch: C equal-shape configurations in one launch pair
+    (the TMA pipeline when L is a multiple of 8, the streaming kernel
+    otherwise), each configuration's [3][N][S] block against the oracle and
+    against its own single-configuration call."""
+    import torch
+    acts, refs = SI.drift_arrays(C * S, N, L, seed=C * 100 + S * 10 + N + L)
+    d_acts = torch.from_numpy(acts.view(np.float16)).cuda()
+    d_refs = torch.from_numpy(refs).cuda()
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    g = cg.cg_drift_scores_batch(d_acts, d_refs, C, S, N, status=st).cpu().numpy()
+    assert cg.cg_read_status(st) == (0, 0)
+    assert g.shape == (3, C, N, S)
+    for c in range(C):
+        a, r = acts[c * S:(c + 1) * S], refs[c * S:(c + 1) * S]
+        assert_scores_close(g[:, c], orc.drift_scores(a, r, S, N), what=f"batch config {c}")
+        if L % 8 == 0:
+            # the TMA pipeline's sums do not depend on where a segment sits,
+            # so a batched configuration scores exactly as it does alone
+            one = cg.cg_drift_scores(d_acts[c * S:(c + 1) * S].clone(),
+                                     d_refs[c * S:(c + 1) * S].clone(), S, N)
+            assert np.array_equal(g[:, c], one.cpu().numpy()), "batch and single call differ"
+
+
+@pytest.mark.parametrize("algo", [1, 2])
+def test_drift_magnitude_domain(cg, orc, algo):
+    """The lower end of the fp32 sums' range (Eq. 4 on tiny activations).
+    References of scale 1e-16 (squares normal) and 1e-20 (squares
+    subnormal, live values fp16(a) = 0, so h - a = -a exactly and D = A
+    term by term) match the oracle: rel_l2 = 1, cos_dev = 0, max_abs exact.
+    At scale 1e-24 every square underflows fp32: the documented result is
+    rel_l2 and cos_dev NaN (the oracle's fp64 gives 1), which the ranking
+    then reports as CG_ERR_NAN_SCORE instead of ranking a wrong value."""
+    import torch
+    S, N, L = 2, 3, 8192
+    rng = np.random.Generator(np.random.PCG64(5))
+    base = rng.standard_normal((S, N, L)).astype(np.float64)
+    scale = np.array([1e-16, 1e-20, 1e-24])[None, :, None]
+    refs = (base * scale).astype(np.float32)
+    acts = refs.astype(np.float16).view(np.uint16)            # fp16 rounds all of them to +-0
+    assert not (acts & 0x7FFF).any()
+    g = run(cg, acts, refs, S, N, algo=algo).cpu().numpy()
+    o = orc.drift_scores(acts, refs, S, N)
+    ok = [0, 1]                                               # canaries of scale 1e-16, 1e-20
+    assert_scores_close(g[:, ok], o[:, ok], what="1e-16 and 1e-20")
+    assert np.all(g[0, ok] == 1.0) and np.all(g[2, ok] == 0.0)
+    assert np.all(np.isnan(g[0, 2])) and np.all(np.isnan(g[2, 2]))
+    assert np.array_equal(g[1, 2], o[1, 2].astype(np.float32))   # max |a| is still exact
+    assert np.all(o[0, 2] == 1.0)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    lab = torch.zeros((1, N, S), dtype=torch.int8, device="cuda")
+    lab[:, :, 0] = 1
+    cg.cg_auroc(torch.from_numpy(g[0]).cuda()[None].contiguous(), lab, status=st)
+    assert cg.cg_read_status(st)[0] == 4                     # CG_ERR_NAN_SCORE
