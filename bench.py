@@ -53,6 +53,7 @@ WORKLOADS = {"70b": SI.SEVENTY_B, "7b": SI.SEVEN_B, "paper_shape": SI.PAPER_SHAP
 METRIC = "canary activation elements scored/sec (HBM GB/s vs peak); AUROC configs/sec"
 BYTES_PER_ELEMENT = 6          # 2 B fp16 live + 4 B fp32 reference, each read once
 L2_BYTES = 129 * 2**20
+NOMINAL_HBM_GBPS = 8000.0      # GB300 HBM3e, nominal
 
 
 def parse_args(argv=None):
@@ -62,7 +63,8 @@ def parse_args(argv=None):
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--workload", default="70b", choices=sorted(WORKLOADS))
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--e2e-steps", type=int, default=25,
+                   help="timed end-to-end steps (25 x ~40 ms: about a second)")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0,
                    help="target duration of the timed CPU-oracle sample")
@@ -479,6 +481,10 @@ def run_ours(args, ranks: Ranks):
             "kernel": drift_kernel + " (+ drift_finalize_kernel inside the same events)",
             "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
             "frac": achieved / peak, "peak_kind": f"{peak_kind} copy bandwidth",
+            # the measured peak is a read+write copy; this kernel only reads, so
+            # its fraction can pass 1.  Beside it, the fraction of the nominal
+            # HBM3e bandwidth the workload targets (about 8 TB/s)
+            "nominal_peak": NOMINAL_HBM_GBPS, "frac_of_nominal": achieved / NOMINAL_HBM_GBPS,
             "traffic": traffic,
             "algorithmic_bytes_per_launch": E * BYTES_PER_ELEMENT,
             "launch_ms_mean": drift_avg_ms, "launch_ms_min": min(drift_ms),
@@ -621,9 +627,11 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
         h_scores.copy_(scores, non_blocking=True)
         h_auroc.copy_(auroc, non_blocking=True)
 
-    ms_copy = timed(step_copy, args.e2e_steps)
+    variant_steps = max(1, min(args.e2e_steps, 10))
+    ms_copy = timed(step_copy, variant_steps)
     out["memcpy_variant"] = {"value": elems / (ms_copy / 1e3), "unit": "elements/s",
                              "h2d_bytes_per_step": h2d, "ms_per_step": ms_copy,
+                             "steps": variant_steps,
                              "link_GBps": h2d / (ms_copy / 1e3) / 1e9,
                              "inputs": "live activations copied with cudaMemcpyAsync, then the "
                                        "device-resident drift pass"}
@@ -635,10 +643,11 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
         refs.copy_(h_refs, non_blocking=True)
         step(i)
 
-    ms2 = timed(step_all, max(1, args.e2e_steps - 1))
+    ms2 = timed(step_all, variant_steps)
     h2d2 = h2d + refs.numel() * refs.element_size()
     out["all_inputs_streamed"] = {"value": elems / (ms2 / 1e3), "unit": "elements/s",
                                   "h2d_bytes_per_step": h2d2, "ms_per_step": ms2,
+                                  "steps": variant_steps,
                                   "link_GBps": h2d2 / (ms2 / 1e3) / 1e9}
     del h_acts, h_refs
     return out
@@ -649,12 +658,47 @@ def run_e2e(cg, torch, dev, stream, acts, refs, labels, S, N, L, args, ranks):
 STUDY_METRIC = "AUROC configs/sec (whole study: generate, score and rank every configuration)"
 
 
-def study_pass(cg, torch, configs, dev, bufs, res, drift_events=None, overlap=True):
-    """Every configuration of a study on the device: generate, drift scores,
-    control labels, per-canary AUROC of rel_l2 / max_abs / cos_dev and of the
-    control, pooled AUROC of rel_l2.  res[c] = those five A-hat values.
+STUDY_BATCH_ELEMENTS = 1 << 29      # elements per drift launch in a study (3.2 GB at 6 B each)
 
-    overlap: configuration c + 1 is generated on one stream while c is scored
+
+def study_batches(configs):
+    """Consecutive runs of configurations with one shape (stages, canaries,
+    segment length) and at most STUDY_BATCH_ELEMENTS elements in all (a
+    larger configuration stands alone).  A run is generated into one buffer
+    and scored by one cg_drift_scores_batch launch pair."""
+    out, key_of_run = [], None
+    for i, c in enumerate(configs):
+        key = (c["n_shards"], c["n_canaries"], c["tokens"] * c["hidden"])
+        if (out and key == key_of_run
+                and (len(out[-1]) + 1) * SI.n_elements(c) <= STUDY_BATCH_ELEMENTS):
+            out[-1].append(i)
+        else:
+            out.append([i])
+            key_of_run = key
+    return out
+
+
+def id_runs(configs, idx):
+    """Split a batch into runs of consecutive config ids: (first position,
+    end position) pairs; one control-label call serves each run."""
+    runs, j = [], 0
+    while j < len(idx):
+        k = j + 1
+        while k < len(idx) and configs[idx[k]]["config_id"] == configs[idx[k - 1]]["config_id"] + 1:
+            k += 1
+        runs.append((j, k))
+        j = k
+    return runs
+
+
+def study_pass(cg, torch, configs, batches, bufs, res, drift_events=None, overlap=True):
+    """Every configuration of a study on the device, one batch of equal-shape
+    configurations at a time: generate each into the batch's buffer, one
+    batched drift launch pair, control labels, per-canary AUROC of rel_l2 /
+    max_abs / cos_dev and of the control, pooled AUROC of rel_l2, each over
+    the whole batch.  res[k, c] = A-hat k of configuration c.
+
+    overlap: batch b + 1 is generated on one stream while batch b is scored
     on another, in alternating pipeline buffers (the generator is bound by
     integer/FP32 issue, the scoring by HBM, and the generator leaves room on
     every SM for a drift block).  The passes fork from and join back into the
@@ -666,46 +710,53 @@ def study_pass(cg, torch, configs, dev, bufs, res, drift_events=None, overlap=Tr
         s_score.wait_stream(main)
     else:
         s_gen = s_score = main
-    for c, cfg in enumerate(configs):
-        S, N, L = cfg["n_shards"], cfg["n_canaries"], cfg["tokens"] * cfg["hidden"]
+    for k, idx in enumerate(batches):
+        c0, B = idx[0], len(idx)
+        cfg0 = configs[c0]
+        S, N, L = cfg0["n_shards"], cfg0["n_canaries"], cfg0["tokens"] * cfg0["hidden"]
         E = S * N * L
-        b = c % 2 if overlap else 0
-        desc = cg.PipelineDesc.from_config(cfg)
-        acts = bufs["acts"][b][:E].view(S, N, L)
-        refs = bufs["refs"][b][:E].view(S, N, L)
-        labels = bufs["labels"][b][:N * S].view(1, N, S)
-        ctrl = bufs["ctrl"][:N * S].view(1, N, S)
+        b = k % 2 if overlap else 0
+        acts = bufs["acts"][b][:B * E].view(B, S, N, L)
+        refs = bufs["refs"][b][:B * E].view(B, S, N, L)
+        labels = bufs["labels"][b][:B * N * S].view(B, N, S)
+        ctrl = bufs["ctrl"][:B * N * S].view(B, N, S)
         with torch.cuda.stream(s_gen):
-            if overlap and c >= 2:
-                s_gen.wait_event(bufs["scored"][b])      # buffer b is free once c - 2 is scored
-            if cfg.get("gain", 0.0):
-                cg.cg_generate_propagating(desc, cfg["gain"], acts, refs, labels[0], bufs["gws"],
-                                           status=bufs["status"])
-            else:
-                cg.cg_generate_pipeline(desc, acts, refs, labels[0], bufs["gws"],
-                                        status=bufs["status"])
+            if overlap and k >= 2:
+                s_gen.wait_event(bufs["scored"][b])      # buffer b is free once batch k - 2 is scored
+            for j, i in enumerate(idx):
+                cfg = configs[i]
+                desc = cg.PipelineDesc.from_config(cfg)
+                if cfg.get("gain", 0.0):
+                    cg.cg_generate_propagating(desc, cfg["gain"], acts[j], refs[j], labels[j],
+                                               bufs["gws"], status=bufs["status"])
+                else:
+                    cg.cg_generate_pipeline(desc, acts[j], refs[j], labels[j], bufs["gws"],
+                                            status=bufs["status"])
             if overlap:
                 bufs["generated"][b].record(s_gen)
         with torch.cuda.stream(s_score):
             if overlap:
                 s_score.wait_event(bufs["generated"][b])
-            scores = bufs["scores"][:3 * N * S].view(3, N, S)
+            scores = bufs["scores"][:3 * B * N * S].view(3, B, N, S)
             if drift_events is not None:
-                drift_events[c][0].record(s_score)
-            cg.cg_drift_scores(acts, refs, S, N, scores=scores, ws=bufs["dws"],
-                               status=bufs["status"])
+                drift_events[k][0].record(s_score)
+            cg.cg_drift_scores_batch(acts, refs, B, S, N, scores=scores, ws=bufs["dws"],
+                                     status=bufs["status"])
             if drift_events is not None:
-                drift_events[c][1].record(s_score)
-            cg.cg_make_control_labels(labels, seed=7000 + c, config_id0=desc.config_id, ctrl=ctrl,
-                                      status=bufs["status"])
-            u2 = bufs["u2"][:N].view(1, N)
-            for k in range(3):
-                cg.cg_auroc(scores[k].view(1, N, S), labels, u2=u2, auroc=res[c, k:k + 1],
+                drift_events[k][1].record(s_score)
+            for j0, j1 in id_runs(configs, idx):
+                cg.cg_make_control_labels(labels[j0:j1], seed=7000,
+                                          config_id0=configs[idx[j0]]["config_id"],
+                                          ctrl=ctrl[j0:j1], status=bufs["status"])
+            u2 = bufs["u2"][:B * N].view(B, N)
+            for st in range(3):
+                cg.cg_auroc(scores[st], labels, u2=u2, auroc=res[st, c0:c0 + B],
                             want_counts=False, status=bufs["status"])
-            cg.cg_auroc(scores[0].view(1, N, S), ctrl, u2=u2, auroc=res[c, 3:4], want_counts=False,
+            cg.cg_auroc(scores[0], ctrl, u2=u2, auroc=res[3, c0:c0 + B], want_counts=False,
                         status=bufs["status"])
-            cg.cg_auroc_pooled(scores[0].view(1, N, S), labels, u2=bufs["pu2"], n_mal=bufs["pnm"],
-                               n_ben=bufs["pnb"], auroc=res[c, 4:5], status=bufs["status"])
+            cg.cg_auroc_pooled(scores[0], labels, u2=bufs["pu2"][:B], n_mal=bufs["pnm"][:B],
+                               n_ben=bufs["pnb"][:B], auroc=res[4, c0:c0 + B],
+                               status=bufs["status"])
             if overlap:
                 bufs["scored"][b].record(s_score)
     if overlap:
@@ -720,14 +771,20 @@ def run_study(args, ranks: Ranks):
     torch.cuda.set_device(ranks.local)
     cg.build()
     configs = [rank_config(c, ranks.rank) for c in SI.STUDIES[args.study]()]
+    batches = study_batches(configs)
     dev = torch.device("cuda", ranks.local)
     stream = torch.cuda.current_stream()
-    maxE = max(SI.n_elements(c) for c in configs)
-    maxNS = max(c["n_canaries"] * c["n_shards"] for c in configs)
-    maxN = max(c["n_canaries"] for c in configs)
+
+    def per_batch(fn):
+        return max(fn(configs[idx[0]], len(idx)) for idx in batches)
+
+    maxE = per_batch(lambda c, B: B * SI.n_elements(c))
+    maxNS = per_batch(lambda c, B: B * c["n_canaries"] * c["n_shards"])
+    maxN = per_batch(lambda c, B: B * c["n_canaries"])
+    maxB = max(len(idx) for idx in batches)
     gws = max(cg.cg_generate_workspace_size(cg.PipelineDesc.from_config(c)) for c in configs)
-    dws = max(cg.cg_drift_workspace_size(c["n_shards"], c["n_canaries"],
-                                         c["tokens"] * c["hidden"]) for c in configs)
+    dws = per_batch(lambda c, B: cg.cg_drift_workspace_size(B * c["n_shards"], c["n_canaries"],
+                                                            c["tokens"] * c["hidden"]))
     bufs = {
         # two pipeline buffers: one being generated while the other is scored
         "acts": [torch.empty(maxE, dtype=torch.float16, device=dev) for _ in range(2)],
@@ -740,16 +797,16 @@ def run_study(args, ranks: Ranks):
         "ctrl": torch.empty(maxNS, dtype=torch.int8, device=dev),
         "scores": torch.empty(3 * maxNS, dtype=torch.float32, device=dev),
         "u2": torch.empty(maxN, dtype=torch.int64, device=dev),
-        "pu2": torch.empty(1, dtype=torch.int64, device=dev),
-        "pnm": torch.empty(1, dtype=torch.int64, device=dev),
-        "pnb": torch.empty(1, dtype=torch.int64, device=dev),
+        "pu2": torch.empty(maxB, dtype=torch.int64, device=dev),
+        "pnm": torch.empty(maxB, dtype=torch.int64, device=dev),
+        "pnb": torch.empty(maxB, dtype=torch.int64, device=dev),
         "gws": torch.empty(gws, dtype=torch.uint8, device=dev),
         "dws": torch.empty(dws, dtype=torch.uint8, device=dev),
         "status": torch.zeros(1, dtype=torch.int32, device=dev),
     }
-    res = torch.empty((len(configs), 5), dtype=torch.float64, device=dev)
+    res = torch.empty((5, len(configs)), dtype=torch.float64, device=dev)
     for _ in range(max(1, args.warmup)):
-        study_pass(cg, torch, configs, dev, bufs, res)
+        study_pass(cg, torch, configs, batches, bufs, res)
     torch.cuda.synchronize()
     clocks = ClockSampler(ranks.local)
     clocks.start()
@@ -758,7 +815,7 @@ def run_study(args, ranks: Ranks):
     reps = max(1, args.steps)
     e0.record(stream)
     for _ in range(reps):
-        study_pass(cg, torch, configs, dev, bufs, res)
+        study_pass(cg, torch, configs, batches, bufs, res)
     e1.record(stream)
     torch.cuda.synchronize()
     ms_eager = ranks.max(e0.elapsed_time(e1)) / reps
@@ -768,7 +825,7 @@ def run_study(args, ranks: Ranks):
     try:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            study_pass(cg, torch, configs, dev, bufs, res)
+            study_pass(cg, torch, configs, batches, bufs, res)
         eager_res = res.clone()
         res.fill_(-1.0)
         g.replay()
@@ -798,16 +855,16 @@ def run_study(args, ranks: Ranks):
     # (one stream, nothing overlapping it); its A-hat values must equal the
     # overlapped passes' bit for bit
     dev_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-              for _ in configs]
+              for _ in batches]
     overlapped_res = res.clone()
-    study_pass(cg, torch, configs, dev, bufs, res, drift_events=dev_ev, overlap=False)
+    study_pass(cg, torch, configs, batches, bufs, res, drift_events=dev_ev, overlap=False)
     torch.cuda.synchronize()
     if not torch.equal(res.view(torch.int64), overlapped_res.view(torch.int64)):
         raise RuntimeError("the overlapped passes' A-hat values differ from the one-stream pass")
     drift_ms = sum(a.elapsed_time(b) for a, b in dev_ev)
     drift_bytes = float(sum(SI.n_elements(c) for c in configs)) * BYTES_PER_ELEMENT
     peak, peak_kind = measured_peaks()
-    A = res.cpu().numpy()
+    A = res.cpu().numpy().T
     total_cfg = ranks.sum(float(len(configs)))
     elems = ranks.sum(float(sum(SI.n_elements(c) for c in configs)))
 
@@ -827,9 +884,12 @@ def run_study(args, ranks: Ranks):
         "data": "synthetic",
         "config": {"workload": f"study '{args.study}': {len(configs)} configurations",
                    "elements_per_pass": elems,
-                   "step": "per configuration: generate (2 to 4 kernels), drift (2), control labels, "
-                           "3 + 1 per-canary AUROC, 1 pooled AUROC; configuration c + 1 is generated "
-                           "on a second stream while c is scored (two pipeline buffers)"},
+                   "batches": len(batches),
+                   "step": "per batch of equal-shape configurations (at most 2^29 elements): "
+                           "generate each (2 to 4 kernels), one batched drift (2), control labels "
+                           "(one call per run of consecutive config ids), 3 + 1 per-canary AUROC "
+                           "and 1 pooled AUROC over the batch; batch b + 1 is generated on a "
+                           "second stream while b is scored (two pipeline buffers)"},
         "elements_per_s": elems / (ms / 1e3),
         "execution": "CUDA graph of one whole pass, replayed" if graph is not None else "eager",
         "eager": {"value": total_cfg / (ms_eager / 1e3), "unit": "configs/s",
@@ -841,32 +901,47 @@ def run_study(args, ranks: Ranks):
         "auroc_summary": summary,
         "per_config_auroc": {n: [round(float(x), 6) for x in A[:, k]] for k, n in enumerate(names)},
         "cpu_baseline": cpu,
-        "gpu_launches": sum(launches_per_config(c) for c in configs) * reps,
+        "gpu_launches": study_launches(configs, batches,
+                                       torch.cuda.get_device_properties(dev).multi_processor_count)
+                        * reps,
         "clocks": clk,
     }
     print(json.dumps(line), flush=True)
 
 
-def auroc_launches(N, S) -> int:
-    """Launches of one cg_auroc call on a single configuration: one block
-    ranks and combines it (S <= 32, N <= 1024), else canary-parallel counts
-    and a per-configuration combine."""
-    return 1 if S <= 32 and N <= 1024 else 2
+def auroc_launches(N, S, C=1, sm_count=152) -> int:
+    """Launches of one cg_auroc call on C configurations: one block per
+    configuration ranks and combines it (S <= 32, N <= 1024), or a warp per
+    configuration (S <= 32, C >= 8 per SM; S > 32, C >= 2 per SM); else
+    canary-parallel counts and a per-configuration combine."""
+    if S <= 32:
+        return 1 if (N <= 1024 or C >= 8 * sm_count) else 2
+    return 1 if C >= 2 * sm_count else 2
 
 
-def launches_per_config(cfg) -> int:
-    """Kernel launches of one study configuration: generator (2 when every
-    stage's live values follow element by element, else 4; 2 + 3 per stage
-    when propagating), drift scores (2), control labels (1), three per-canary
-    AUROC calls and the control's, pooled AUROC (1)."""
+def generator_launches(cfg) -> int:
+    """Generator kernels of one configuration: 2 when every stage's live values
+    follow element by element, else 4; 2 + 3 per stage when propagating."""
     if cfg.get("gain", 0.0):
-        gen = 2 + 3 * cfg["n_shards"]
-    else:
-        n_mal = len(cfg["malicious"])
-        needs_stats = ((n_mal < cfg["n_shards"] and cfg["noise"] == SI.NOISE_PAPER) or
-                       (n_mal > 0 and cfg["tamper"] == SI.TAMPER_ADDITIVE))
-        gen = 4 if needs_stats else 2
-    return gen + 2 + 1 + 4 * auroc_launches(cfg["n_canaries"], cfg["n_shards"]) + 1
+        return 2 + 3 * cfg["n_shards"]
+    n_mal = len(cfg["malicious"])
+    needs_stats = ((n_mal < cfg["n_shards"] and cfg["noise"] == SI.NOISE_PAPER) or
+                   (n_mal > 0 and cfg["tamper"] == SI.TAMPER_ADDITIVE))
+    return 4 if needs_stats else 2
+
+
+def study_launches(configs, batches, sm_count=152) -> int:
+    """Kernel launches of one study pass: per batch, every configuration's
+    generator, the batched drift (2), one control-label call per run of
+    consecutive ids, three per-canary AUROC calls and the control's, and
+    the pooled AUROC (1)."""
+    total = 0
+    for idx in batches:
+        c, B = configs[idx[0]], len(idx)
+        total += sum(generator_launches(configs[i]) for i in idx)
+        total += 2 + len(id_runs(configs, idx)) + 1
+        total += 4 * auroc_launches(c["n_canaries"], c["n_shards"], B, sm_count)
+    return total
 
 
 def study_oracle_baseline(cfgs, seconds):
