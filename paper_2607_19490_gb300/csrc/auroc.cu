@@ -248,29 +248,54 @@ __device__ __forceinline__ uint32_t zero_byte_flags(uint32_t x) {
   return ~(((x & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | x) & 0x80808080u;
 }
 
+// The stage k whose mask bit is i (the inverse of stage_bit for S <= 32).
+__device__ __forceinline__ int stage_of_bit(int i) { return 4 * (i & 7) + (i >> 3); }
+
+// m[k] for a run-time k without dynamic register indexing: a tree of
+// selects on the bits of k, low bit first (SP - 1 selects).
+template <int SP>
+__device__ __forceinline__ float select_stage(const float (&m)[SP], int k) {
+  float t[SP];
+#pragma unroll
+  for (int j = 0; j < SP; ++j) t[j] = m[j];
+#pragma unroll
+  for (int half = SP / 2, bit = 0; half >= 1; half /= 2, ++bit) {
+    const bool odd = (k >> bit) & 1;
+#pragma unroll
+    for (int j = 0; j < half; ++j) t[j] = odd ? t[2 * j + 1] : t[2 * j];
+  }
+  return t[0];
+}
+
 template <int SP>
 __device__ __forceinline__ void lane_rank(const LaneRow<SP> &r, int &g, int &e, int &nm, int &nb,
                                           bool &saw_nan) {
-  uint32_t mal = 0u, ben = 0u, nan = 0u;
+  uint32_t mal = 0u, ben = 0u;
 #pragma unroll
   for (int w = 0; w < SP / 4; ++w) {
     ben |= zero_byte_flags(r.lw[w]) >> (7 - w);                 // label 0
     mal |= zero_byte_flags(r.lw[w] ^ 0x01010101u) >> (7 - w);   // label 1
   }
+  // a NaN anywhere in the row (one unordered compare per stage); only then
+  // are the NaN stages matched against the labelled ones
+  bool any_nan = false;
 #pragma unroll
-  for (int k = 0; k < SP; ++k) nan |= (uint32_t)is_nan_f(r.m[k]) << stage_bit(k);
-  if (nan & (mal | ben)) saw_nan = true;
+  for (int k = 0; k < SP; ++k) any_nan |= is_nan_f(r.m[k]);
+  if (any_nan) {
+    uint32_t nan = 0u;
+#pragma unroll
+    for (int k = 0; k < SP; ++k) nan |= (uint32_t)is_nan_f(r.m[k]) << stage_bit(k);
+    if (nan & (mal | ben)) saw_nan = true;
+  }
   nm = __popc(mal);
   nb = __popc(ben);
   int lg = 0, le = 0;
-  // only the malicious stages are walked; m_i is picked by selects (no
-  // dynamic register indexing) and compared with every stage at once
+  // only the malicious stages are walked; m_i is picked by a select tree
+  // and compared with every stage at once
   while (mal) {
     const int i = __ffs(mal) - 1;
     mal &= mal - 1u;
-    float mi = 0.f;
-#pragma unroll
-    for (int k = 0; k < SP; ++k) mi = (stage_bit(k) == i) ? r.m[k] : mi;
+    const float mi = select_stage<SP>(r.m, stage_of_bit(i));
     uint32_t gtm = 0u, eqm = 0u;
 #pragma unroll
     for (int j = 0; j < SP; ++j) {
