@@ -524,6 +524,15 @@ def auroc_batches(cg, torch, dev, stream):
         ms = e0.elapsed_time(e1) / reps
         out[f"{name}_configs_per_s"] = C / (ms / 1e3)
         out[f"{name}_ms"] = ms
+        if name == "stress_batch":
+            # algorithmic bytes: every score (4 B) and label (1 B) read once,
+            # u2 (8 B per canary) and A-hat (8 B per configuration) written
+            read = C * N * S * 5
+            written = C * N * 8 + C * 8
+            peak, _ = measured_peaks()
+            out["stress_batch_read_GBps"] = read / (ms / 1e3) / 1e9
+            out["stress_batch_GBps"] = (read + written) / (ms / 1e3) / 1e9
+            out["stress_batch_frac"] = (read + written) / (ms / 1e3) / 1e9 / peak
         if name == "factorial_batch":
             # the same call replayed from a CUDA graph: the kernels' own time,
             # without the host's per-call cost
