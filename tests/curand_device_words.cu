@@ -2,7 +2,8 @@
 // GPU) for a few (seed, subsequence, offset) triples, one line per triple:
 //   seed subsequence offset w0 w1 w2 w3 w4 w5 w6 w7
 // Used by tests/test_gpu_curand_pin.py to pin the oracle's Philox counter
-// words 2 and 3 (the subsequence) independently of this repository's code.
+// words 2 and 3 (the subsequence) and, through offsets beyond 4 * 2^32,
+// word 1 independently of this repository's code.
 #include <cstdio>
 #include <cstdint>
 #include <curand_kernel.h>
@@ -19,7 +20,12 @@ int main() {
   const unsigned long long cases[][3] = {
       {0ull, 0ull, 0ull},         {0x123456789ABCDEF0ull, 5ull, 0ull},
       {42ull, 1ull << 32, 0ull},  {42ull, (3ull << 32) | 17ull, 0ull},
-      {7ull, (1ull << 33) + 1234, 4ull * 1000},  {2ull, 0xFFFFFFFF00000003ull, 8ull}};
+      {7ull, (1ull << 33) + 1234, 4ull * 1000},  {2ull, 0xFFFFFFFF00000003ull, 8ull},
+      // offsets past 4 * 2^32 carry into counter word 1; these reach the
+      // auxiliary streams' word 1 = (purpose << 24) | sub
+      {5ull, 9ull, 4ull * ((1ull << 32) * ((1ull << 24) | 3ull) + 100ull)},
+      {11ull, (4ull << 32) | 2ull, 4ull * ((1ull << 32) * ((4ull << 24) | 77ull) + 7ull)},
+      {13ull, 3ull, 4ull * ((1ull << 32) * ((5ull << 24) | 0xFFFFFFull))}};
   const int n = sizeof(cases) / sizeof(cases[0]);
   unsigned long long *d_args;
   unsigned int *d_out;
@@ -27,7 +33,7 @@ int main() {
   if (cudaMalloc(&d_out, n * 8 * sizeof(unsigned int)) != cudaSuccess) return 1;
   cudaMemcpy(d_args, cases, sizeof(cases), cudaMemcpyHostToDevice);
   words<<<1, 32>>>(d_args, n, d_out);
-  unsigned int out[64];
+  unsigned int out[8 * 16];
   if (cudaMemcpy(out, d_out, n * 8 * sizeof(unsigned int), cudaMemcpyDeviceToHost) != cudaSuccess)
     return 1;
   for (int i = 0; i < n; ++i) {
