@@ -162,37 +162,43 @@ drift_partial_kernel(const uint16_t *__restrict__ acts, const float *__restrict_
 //             (D - E^2 / (sqrt H + sqrt A)^2) / (2 sqrt(H A)), which equals
 //             (D - (sqrt H - sqrt A)^2) / (2 sqrt(H A)) without cancelling
 //             two near-equal norms.
-// One warp per segment: lane l adds the items l, l + 32, ... in order in
-// fp64, then a fixed shuffle tree combines the lanes.  Segment
+// G = 2^log_g lanes per segment (the smallest power of two that leaves each
+// lane at most 8 items, at most 32): lane l of the group adds the items
+// l, l + G, ... in order in fp64, then a fixed shuffle tree combines the
+// group.  A segment of few items thus takes few lanes (3 items: one lane, so
+// a warp finishes 32 segments), and a long one a whole warp.  Segment
 // q = (c S + s) N + n of C configurations writes its scores at
 // stat * stat_stride + c N S + n S + s.
 constexpr int kFinThreads = 256;
 
 __global__ void __launch_bounds__(kFinThreads)
 drift_finalize_kernel(const float4 *__restrict__ partials, uint64_t chunks_per_seg, uint32_t C,
-                      uint32_t S, uint32_t N, float *__restrict__ scores, uint64_t stat_stride) {
-  const uint64_t seg = ((uint64_t)blockIdx.x * kFinThreads + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
+                      uint32_t S, uint32_t N, float *__restrict__ scores, uint64_t stat_stride,
+                      int log_g) {
+  const int G = 1 << log_g;
+  const uint64_t seg = ((uint64_t)blockIdx.x * kFinThreads + threadIdx.x) >> log_g;
+  const int sub = threadIdx.x & (G - 1);
   const uint64_t per_config = (uint64_t)S * N;
-  if (seg >= (uint64_t)C * per_config) return;   // whole warps leave together
+  const bool live = seg < (uint64_t)C * per_config;
   double D = 0.0, E = 0.0, A = 0.0;
   float M = 0.f;
-  const float4 *p = partials + seg * chunks_per_seg;
-  for (uint64_t c = lane; c < chunks_per_seg; c += 32) {
-    const float4 v = p[c];
-    D += (double)v.x;
-    E += (double)v.y;
-    A += (double)v.z;
-    M = fmaxf(M, v.w);
+  if (live) {
+    const float4 *p = partials + seg * chunks_per_seg;
+    for (uint64_t c = sub; c < chunks_per_seg; c += G) {
+      const float4 v = p[c];
+      D += (double)v.x;
+      E += (double)v.y;
+      A += (double)v.z;
+      M = fmaxf(M, v.w);
+    }
   }
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) {
-    D += __shfl_down_sync(0xFFFFFFFFu, D, off);
-    E += __shfl_down_sync(0xFFFFFFFFu, E, off);
-    A += __shfl_down_sync(0xFFFFFFFFu, A, off);
-    M = fmaxf(M, __shfl_down_sync(0xFFFFFFFFu, M, off));
+  for (int off = G >> 1; off > 0; off >>= 1) {
+    D += __shfl_down_sync(0xFFFFFFFFu, D, off, G);
+    E += __shfl_down_sync(0xFFFFFFFFu, E, off, G);
+    A += __shfl_down_sync(0xFFFFFFFFu, A, off, G);
+    M = fmaxf(M, __shfl_down_sync(0xFFFFFFFFu, M, off, G));
   }
-  if (lane != 0) return;
+  if (!live || sub != 0) return;
   // The sums stay fp64; the scores are formed in fp32 from them (GB300's
   // FP64 pipe is narrow, and fp32 sqrt/div of the rounded sums is accurate
   // to a few 1e-7 relative, far inside the drift tolerances).
@@ -234,9 +240,11 @@ static cudaError_t launch_finalize(const float4 *partials, uint64_t cps, uint32_
                                    uint32_t N, float *scores, uint64_t stat_stride,
                                    cudaStream_t stream) {
   const uint64_t n_seg = (uint64_t)C * S * N;
-  const uint64_t blocks = (n_seg * 32 + kFinThreads - 1) / kFinThreads;
+  int log_g = 0;                                   // lanes per segment: 2^log_g
+  while (log_g < 5 && ((uint64_t)8 << log_g) < cps) ++log_g;
+  const uint64_t blocks = ((n_seg << log_g) + kFinThreads - 1) / kFinThreads;
   drift_finalize_kernel<<<(unsigned)blocks, kFinThreads, 0, stream>>>(partials, cps, C, S, N,
-                                                                      scores, stat_stride);
+                                                                      scores, stat_stride, log_g);
   return cudaGetLastError();
 }
 
