@@ -75,6 +75,29 @@ def test_auroc_batched_lanes_match_oracle(cg, orc, C, N, S, n_mal, excluded, tie
     assert np.array_equal(g["auroc"][fin].view(np.uint64), o["auroc"][fin].view(np.uint64))
 
 
+@pytest.mark.parametrize("C,N,S,n_mal,excluded,ties", [
+    (1216, 64, 16, 1, 0, None), (1300, 4, 4, 1, 0, 2), (1250, 36, 8, 2, 1, 3),
+    (1230, 50, 32, 5, 3, None), (1290, 2, 8, 1, 0, None), (1217, 33, 16, 3, 2, 4),
+    (3001, 64, 16, 2, 1, 5),
+])
+def test_auroc_many_small_configurations(cg, orc, C, N, S, n_mal, excluded, ties):
+    """Batches of at least 8 configurations per SM with rows of exactly SP
+    stages and at most 64 canaries (a warp per configuration, 16-byte row
+    loads): every SP, a single canary pair, ties, excluded stages,
+    non-uniform pair counts and a configuration without any pair."""
+    scores, labels = SI.score_arrays(C, N, S, seed=C + 5 * N + S, n_malicious=n_mal,
+                                     tie_levels=ties, excluded=excluded)
+    labels[7, ::3, :] = np.where(labels[7, ::3, :] == 0, -1, labels[7, ::3, :])   # fewer pairs
+    labels[11, :, :] = 0                                                          # no pair
+    g = run(cg, scores, labels)
+    o = orc.auroc(scores, labels)
+    for k in ("u2", "gt", "eq"):
+        assert np.array_equal(g[k], o[k]), k
+    fin = ~np.isnan(o["auroc"])
+    assert not fin[11] and np.isnan(g["auroc"][11])
+    assert np.array_equal(g["auroc"][fin].view(np.uint64), o["auroc"][fin].view(np.uint64))
+
+
 def test_auroc_stress_batch(cg, orc):
     """65,536 configurations x 64 canaries x 16 stages."""
     rng = np.random.Generator(np.random.PCG64(5))
@@ -152,8 +175,10 @@ def test_pooled_nan_flag(cg, orc):
     assert np.array_equal(g["u2"].cpu().numpy(), o["u2"])
 
 
-@pytest.mark.parametrize("C,N,S", [(2, 5, 8), (1300, 8, 16), (2, 3, 40), (1300, 33, 4)],
-                         ids=["block", "lane_config", "wide", "lane_config_S4"])
+@pytest.mark.parametrize("C,N,S", [(2, 5, 8), (1300, 8, 16), (1300, 65, 16), (2, 3, 40),
+                                   (1300, 33, 4), (1300, 36, 8)],
+                         ids=["block", "lane_config", "lane_config_N65", "wide", "lane_config_S4",
+                              "lane_config_S8"])
 def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
     """A NaN score on a stage the labels exclude (-1) is not part of any pair:
     no NaN flag, and counts and A-hat equal the oracle's, on every kernel
@@ -176,8 +201,8 @@ def test_nan_on_excluded_stages_is_ignored(cg, orc, C, N, S):
     assert np.array_equal(gp["auroc"].cpu().numpy().view(np.uint64), op["auroc"].view(np.uint64))
 
 
-@pytest.mark.parametrize("C,N,S", [(3, 40, 8), (1300, 8, 16), (2, 6, 40)],
-                         ids=["block", "lane_config", "wide"])
+@pytest.mark.parametrize("C,N,S", [(3, 40, 8), (1300, 8, 16), (1300, 70, 16), (2, 6, 40)],
+                         ids=["block", "lane_config", "lane_config_N70", "wide"])
 def test_auroc_infinities_and_signed_zero(cg, orc, C, N, S):
     """Scores of +inf (a drift score of an infinite activation), -inf, +0 and
     -0 (equal, a tie) among finite ones: counts and A-hat equal the oracle's
