@@ -2,12 +2,17 @@
  * Plain C client of the canary_guard C ABI (no Python, no torch): generate
  * the tiny synthetic pipeline on the device, score every (stage, canary)
  * segment, draw the scrambled-label control and rank both label sets.
- * Prints "A_hat <value> control <value> status <code>" and exits 0 on
- * success.  Built and run by tests/test_gpu_c_client.py.
+ * Then scores a batch of two configurations in one call (the first the
+ * same pipeline) and the first configuration without a workspace, and
+ * compares both with the single call.  Prints "A_hat <value> control
+ * <value> status <code> batch_equal <0|1> noalloc_close <0|1>" and exits 0
+ * on success.  Built and run by tests/test_gpu_c_client.py.
  */
 #include <cuda_runtime_api.h>
+#include <math.h>
 #include <stdint.h>
 #include <stdio.h>
+#include <string.h>
 
 #include "canary_guard.h"
 
@@ -70,9 +75,48 @@ int main(void) {
   cg_status st = cg_read_status(status, stream, &word);
   double a[2];
   CHECK_CUDA(cudaMemcpy(a, auroc, sizeof(a), cudaMemcpyDeviceToHost));
-  printf("A_hat %.6f control %.6f status %d\n", a[0], a[1], (int)st);
+
+  /* a batch of two configurations: [2][S][N][L], the first this pipeline */
+  uint16_t *acts2; float *refs2, *scores2, *scores3; void *dws2;
+  size_t drift_ws2 = 0;
+  CHECK_CG(cg_drift_workspace_size(2 * d.n_shards, d.n_canaries, L, &drift_ws2));
+  CHECK_CUDA(cudaMalloc((void **)&acts2, 2 * S * N * L * 2));
+  CHECK_CUDA(cudaMalloc((void **)&refs2, 2 * S * N * L * 4));
+  CHECK_CUDA(cudaMalloc((void **)&scores2, 3 * 2 * N * S * 4));
+  CHECK_CUDA(cudaMalloc((void **)&scores3, 3 * N * S * 4));
+  CHECK_CUDA(cudaMalloc(&dws2, drift_ws2));
+  cg_pipeline_desc d1 = d;
+  d1.config_id = 1;
+  CHECK_CG(cg_generate_pipeline(&d, acts2, refs2, NULL, gws, gen_ws, status, stream));
+  CHECK_CG(cg_generate_pipeline(&d1, acts2 + S * N * L, refs2 + S * N * L, NULL, gws, gen_ws,
+                                status, stream));
+  CHECK_CG(cg_drift_scores_batch(acts2, refs2, 2, d.n_shards, d.n_canaries, L, scores2,
+                                 2 * N * S, dws2, drift_ws2, status, stream));
+  CHECK_CG(cg_drift_scores_noalloc(acts, refs, d.n_shards, d.n_canaries, L, scores3, N * S,
+                                   status, stream));
+  float one[3 * 16 * 4], two[3 * 2 * 16 * 4], na[3 * 16 * 4];
+  CHECK_CUDA(cudaMemcpy(one, scores, sizeof(one), cudaMemcpyDeviceToHost));
+  CHECK_CUDA(cudaMemcpy(two, scores2, sizeof(two), cudaMemcpyDeviceToHost));
+  CHECK_CUDA(cudaMemcpy(na, scores3, sizeof(na), cudaMemcpyDeviceToHost));
+  int batch_equal = 1, noalloc_close = 1;
+  for (size_t k = 0; k < 3; ++k)
+    for (size_t i = 0; i < N * S; ++i) {
+      /* configuration 0 of the batch: the same bytes as the single call */
+      if (memcmp(&one[k * N * S + i], &two[k * 2 * N * S + i], sizeof(float)) != 0)
+        batch_equal = 0;
+      /* the no-workspace call streams through registers: its fp32 sums are
+         added in another order, so rel_l2 within 1e-5 relative, cos_dev
+         within 1e-5 of max(cos_dev, rel_l2^2 / 2), max_abs exact */
+      const float x = one[k * N * S + i], y = na[k * N * S + i], m = one[i];
+      const float scale = k == 2 ? fmaxf(fabsf(x), 0.5f * m * m) : fabsf(x);
+      if (k == 1 ? x != y : fabsf(x - y) > 1e-5f * scale + 1e-12f) noalloc_close = 0;
+    }
+  if (cg_read_status(status, stream, &word) != CG_OK) st = CG_ERR_TIMEOUT;
+  printf("A_hat %.6f control %.6f status %d batch_equal %d noalloc_close %d\n", a[0], a[1],
+         (int)st, batch_equal, noalloc_close);
 
   cudaFree(acts); cudaFree(refs); cudaFree(scores); cudaFree(labels); cudaFree(ctrl);
   cudaFree(gws); cudaFree(dws); cudaFree(u2); cudaFree(auroc); cudaFree(status);
-  return st == CG_OK ? 0 : 1;
+  cudaFree(acts2); cudaFree(refs2); cudaFree(scores2); cudaFree(scores3); cudaFree(dws2);
+  return (st == CG_OK && batch_equal && noalloc_close) ? 0 : 1;
 }
