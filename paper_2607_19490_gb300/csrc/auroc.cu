@@ -781,6 +781,180 @@ auroc_pooled_kernel(const float *__restrict__ scores, const int8_t *__restrict__
     atomicOr(status, CG_DEVFLAG_NAN_SCORE);
 }
 
+// Pairs of the larger side against the sorted, padded smaller side of
+// M = 2^LOG keys: for each larger-side key v (lane-strided), the lower and
+// upper bounds of v in `sorted` by LOG unrolled halving steps each, both
+// searches interleaved; gt and eq as in auroc_pooled_kernel.
+template <int LOG>
+__device__ __forceinline__ void pool_count(const uint32_t *sorted, const uint32_t *large,
+                                           uint32_t nl, uint32_t ns, bool small_mal, int lane,
+                                           uint32_t &gt, uint32_t &eq) {
+  for (uint32_t i = lane; i < nl; i += 32) {
+    const uint32_t v = large[i];
+    uint32_t pl = 0u, ph = 0u;
+#pragma unroll
+    for (int b = LOG - 1; b >= 0; --b) {
+      const uint32_t step = 1u << b;
+      const uint32_t xl = sorted[pl + step - 1], xh = sorted[ph + step - 1];
+      pl += (xl < v) ? step : 0u;
+      ph += (xh <= v) ? step : 0u;
+    }
+    const uint32_t lo = pl + (sorted[pl] < v ? 1u : 0u);
+    const uint32_t hi = ph + (sorted[ph] <= v ? 1u : 0u);
+    gt += small_mal ? (ns - hi) : lo;
+    eq += hi - lo;
+  }
+}
+
+// Pooled Mann-Whitney with one warp per configuration, for configurations
+// of at most kPoolWarpMaxPer scores: the same compaction, sort of the
+// smaller side and bound searches as auroc_pooled_kernel, but each warp
+// works in its own part of shared memory and synchronises only itself, so
+// the eight warps of a block rank eight configurations at once with no
+// block-wide barrier and no shared atomics.  The smaller side holds at most
+// per / 2 keys: up to 64 they are sorted in registers (warp_sort64), above
+// that by a warp bitonic sort in shared memory.  Counts fit 32 bits
+// (n_mal n_ben <= 512^2).
+constexpr uint32_t kPoolWarpMaxPer = 1024;
+constexpr uint32_t kPoolWarpMaxSmall = kPoolWarpMaxPer / 2;
+constexpr size_t kPoolWarpSmem = (size_t)kPoolWarps * (kPoolWarpMaxPer + kPoolWarpMaxSmall) * 4;
+
+__global__ void __launch_bounds__(kPoolThreads)
+auroc_pooled_warp_kernel(const float *__restrict__ scores, const int8_t *__restrict__ labels,
+                         uint32_t C, uint32_t per, bool vec, int64_t *__restrict__ u2_out,
+                         int64_t *__restrict__ nm_out, int64_t *__restrict__ nb_out,
+                         double *__restrict__ auroc, int32_t *status) {
+  extern __shared__ uint32_t pw_smem[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t *keys = pw_smem + (size_t)warp * (kPoolWarpMaxPer + kPoolWarpMaxSmall);
+  uint32_t *sorted = keys + kPoolWarpMaxPer;
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  bool nan_seen = false;
+  const uint64_t warps = (uint64_t)gridDim.x * kPoolWarps;
+  for (uint64_t c = (uint64_t)blockIdx.x * kPoolWarps + warp; c < C; c += warps) {
+    const float *m = scores + c * per;
+    const int8_t *l = labels + c * per;
+    // labelled scores -> order-preserving keys: malicious from the front,
+    // benign from the back (the order inside each side does not matter)
+    uint32_t nm = 0u, nb = 0u;                       // warp-uniform counts so far
+    auto place = [&](int lab, float x) {
+      if (lab == 0 || lab == 1) {
+        if (is_nan_f(x)) {
+          nan_seen = true;
+          lab = -1;
+        }
+      } else {
+        lab = -1;
+      }
+      const uint32_t mal = __ballot_sync(0xFFFFFFFFu, lab == 1);
+      const uint32_t ben = __ballot_sync(0xFFFFFFFFu, lab == 0);
+      if (lab == 1) keys[nm + __popc(mal & lt_mask)] = order_key(x);
+      else if (lab == 0) keys[per - 1u - (nb + __popc(ben & lt_mask))] = order_key(x);
+      nm += __popc(mal);
+      nb += __popc(ben);
+    };
+    if (vec) {
+      // 4 scores (16 bytes) and 4 labels (4 bytes) per lane and load, 4 loads
+      // of each in flight before any is placed
+      constexpr int U = 4;
+      for (uint32_t i0 = 0; i0 < per; i0 += 128u * U) {
+        float4 xv[U];
+        uint32_t lv[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          const uint32_t i = i0 + 128u * u + 4u * (uint32_t)lane;
+          if (i < per) {
+            xv[u] = *reinterpret_cast<const float4 *>(m + i);
+            lv[u] = *reinterpret_cast<const uint32_t *>(l + i);
+          } else {
+            xv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            lv[u] = 0xFFFFFFFFu;                     // -1: left out
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          place((int)(int8_t)(lv[u] & 0xFFu), xv[u].x);
+          place((int)(int8_t)((lv[u] >> 8) & 0xFFu), xv[u].y);
+          place((int)(int8_t)((lv[u] >> 16) & 0xFFu), xv[u].z);
+          place((int)(int8_t)(lv[u] >> 24), xv[u].w);
+        }
+      }
+    } else {
+      for (uint32_t i0 = 0; i0 < per; i0 += 32) {
+        const uint32_t i = i0 + (uint32_t)lane;
+        int lab = -1;
+        float x = 0.f;
+        if (i < per) {
+          lab = l[i];
+          if (lab == 0 || lab == 1) x = m[i];
+        }
+        place(lab, x);
+      }
+    }
+    __syncwarp();
+    const bool small_mal = nm <= nb;
+    const uint32_t ns = small_mal ? nm : nb, nl = small_mal ? nb : nm;
+    const uint32_t *small = small_mal ? keys : keys + (per - nb);
+    const uint32_t *large = small_mal ? keys + (per - nb) : keys;
+    uint32_t M = 1;
+    while (M < ns) M <<= 1;
+    if (M <= 64) {
+      uint32_t r0 = (uint32_t)lane < ns ? small[lane] : 0xFFFFFFFFu;
+      uint32_t r1 = (uint32_t)lane + 32u < ns ? small[lane + 32] : 0xFFFFFFFFu;
+      warp_sort64(r0, r1, M, lane);
+      if ((uint32_t)lane < M) sorted[lane] = r0;
+      if ((uint32_t)lane + 32u < M) sorted[lane + 32] = r1;
+    } else {
+      for (uint32_t i = lane; i < M; i += 32) sorted[i] = i < ns ? small[i] : 0xFFFFFFFFu;
+      __syncwarp();
+      for (uint32_t k = 2; k <= M; k <<= 1) {
+        for (uint32_t j = k >> 1; j > 0; j >>= 1) {
+          for (uint32_t i = lane; i < M; i += 32) {
+            const uint32_t ixj = i ^ j;
+            if (ixj > i) {
+              const uint32_t a = sorted[i], b = sorted[ixj];
+              if ((a > b) == ((i & k) == 0)) {
+                sorted[i] = b;
+                sorted[ixj] = a;
+              }
+            }
+          }
+          __syncwarp();
+        }
+      }
+    }
+    __syncwarp();
+    uint32_t gt = 0u, eq = 0u;
+    if (ns > 0) {
+      switch (31 - __clz(M)) {                      // log2 M, 0 .. 9
+        case 0: pool_count<0>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 1: pool_count<1>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 2: pool_count<2>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 3: pool_count<3>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 4: pool_count<4>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 5: pool_count<5>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 6: pool_count<6>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 7: pool_count<7>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        case 8: pool_count<8>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+        default: pool_count<9>(sorted, large, nl, ns, small_mal, lane, gt, eq); break;
+      }
+    }
+    gt = __reduce_add_sync(0xFFFFFFFFu, gt);
+    eq = __reduce_add_sync(0xFFFFFFFFu, eq);
+    if (lane == 0) {
+      const long long u2 = 2ll * (long long)gt + (long long)eq;
+      const long long NM = nm, NB = nb;
+      u2_out[c] = u2;
+      if (nm_out) nm_out[c] = NM;
+      if (nb_out) nb_out[c] = NB;
+      auroc[c] = (NM * NB > 0) ? __ddiv_rn((double)u2, (double)(2 * NM * NB)) : NAN;
+    }
+    __syncwarp();   // keys and sorted are rewritten by the next configuration
+  }
+  if (__any_sync(0xFFFFFFFFu, nan_seen) && lane == 0 && status)
+    atomicOr(status, CG_DEVFLAG_NAN_SCORE);
+}
+
 }  // namespace
 
 cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint32_t C,
@@ -790,6 +964,23 @@ cudaError_t launch_auroc_pooled(const float *scores, const int8_t *labels, uint3
   DeviceInfo info;
   if (!device_info(&info)) return cudaGetLastError();
   const uint32_t per = N * S;
+  if (per <= kPoolWarpMaxPer) {
+    // a warp per configuration, eight per block, the blocks that fit at once
+    uint64_t grid = ((uint64_t)C + kPoolWarps - 1) / kPoolWarps;
+    int occ = 0;
+    cudaError_t err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &occ, auroc_pooled_warp_kernel, kPoolThreads, kPoolWarpSmem);
+    if (err != cudaSuccess) return err;
+    const uint64_t resident = (uint64_t)info.sm_count * (uint64_t)(occ > 0 ? occ : 1);
+    if (grid > resident) grid = resident;
+    // 16-byte score and 4-byte label loads when every configuration's row
+    // starts on those boundaries
+    const bool vec = (per % 4) == 0 && ((uintptr_t)scores % 16) == 0 &&
+                     ((uintptr_t)labels % 4) == 0;
+    auroc_pooled_warp_kernel<<<(unsigned)grid, kPoolThreads, kPoolWarpSmem, stream>>>(
+        scores, labels, C, per, vec, u2, n_mal, n_ben, auroc, status);
+    return cudaGetLastError();
+  }
   uint32_t Ms = 1;                                // the smaller side holds at most per / 2 keys
   while (Ms < (per + 1) / 2) Ms <<= 1;
   const size_t smem = (size_t)(per + Ms) * sizeof(uint32_t);

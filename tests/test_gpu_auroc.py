@@ -142,6 +142,9 @@ def test_control_no_benign_flag(cg):
     (1, 1, 2, 1, 0, None), (5, 7, 4, 1, 0, None), (3, 64, 16, 1, 0, 3), (4, 9, 32, 3, 2, 5),
     (2, 256, 16, 1, 0, None), (2, 1000, 16, 2, 1, 7), (324, 64, 16, 1, 0, None), (1, 1, 1000, 10, 3, 6),
     (6, 50, 4, 3, 0, 3), (1, 1024, 16, 9, 0, 4), (1000, 32, 8, 5, 1, 3), (2, 16, 8, 2, 0, 1),
+    # a warp per configuration (N S <= 1024) with a smaller side above 64 keys
+    # (the shared-memory bitonic sort): 512 against 512, and a ragged 1023
+    (50, 64, 16, 8, 0, None), (7, 33, 31, 13, 2, 9), (1300, 64, 16, 8, 0, 5),
 ])
 def test_pooled_matches_oracle(cg, orc, C, N, S, n_mal, excluded, ties):
     import torch
