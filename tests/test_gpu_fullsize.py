@@ -52,7 +52,7 @@ def test_workload_matches_oracle_at_full_size(cg, orc, name):
     import torch
     cfg = WORKLOADS[name]()
     t0 = time.perf_counter()
-    g = run_gpu(cg, cfg, algos=(cg.DRIFT_STREAM, cg.DRIFT_BULK_2CTA))
+    g = run_gpu(cg, cfg, algos=(cg.DRIFT_STREAM, cg.DRIFT_BULK, cg.DRIFT_BULK_2CTA))
     torch.cuda.synchronize()
     out = check_against_oracle(orc, cfg, g)
     if name in EXPECTED_REL_L2:
