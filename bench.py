@@ -553,8 +553,8 @@ def auroc_batches(cg, torch, dev, stream):
             except Exception as exc:       # capture unsupported here: the eager figure stands
                 out[f"{name}_graph_error"] = f"{type(exc).__name__}: {exc}"[:200]
         if name == "stress_batch":
-            # the pooled Mann-Whitney (f2): one block-wide bitonic sort of the
-            # N * S labelled scores per configuration
+            # the pooled Mann-Whitney statistic: per configuration the smaller
+            # side's keys sorted, the larger side's bound-searched in them
             pu = {k: torch.empty((C,), dtype=torch.int64, device=dev) for k in ("u2", "nm", "nb")}
             pa = torch.empty((C,), dtype=torch.float64, device=dev)
             for _ in range(3):
@@ -570,6 +570,20 @@ def auroc_batches(cg, torch, dev, stream):
             out["pooled_stress_batch_configs_per_s"] = C / (pms / 1e3)
             out["pooled_stress_batch_ms"] = pms
             out["pooled_stress_batch_read_GBps"] = C * N * S * 5 / (pms / 1e3) / 1e9
+            # the random baseline's scores (Sec. 4.5) of the same shape: one
+            # Philox block per four scores, 4 B written per score
+            rs = torch.empty_like(scores)
+            for _ in range(3):
+                cg.cg_random_scores(11, C, N, S, out=rs)
+            e0.record(stream)
+            for _ in range(reps):
+                cg.cg_random_scores(11, C, N, S, out=rs)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            rms = e0.elapsed_time(e1) / reps
+            out["random_scores_stress_batch_ms"] = rms
+            out["random_scores_stress_batch_write_GBps"] = C * N * S * 4 / (rms / 1e3) / 1e9
+            del rs
         del scores, labels
     return out
 

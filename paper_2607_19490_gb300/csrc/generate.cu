@@ -542,17 +542,62 @@ gen_prop_live_kernel(GenParams p, uint32_t s, float gain, const uint32_t *__rest
 }
 
 // ----------------------------------------------------------------- random baseline
-// Sec. 4.5: every score replaced by Uniform(0, 1).  Thread per (config,
-// canary); score s = (x >> 8) 2^-24 with x word s of aux stream
-// (RANDOM, canary) of config id config_id0 + c.
-__global__ void random_scores_kernel(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
-                                     uint32_t S, float *__restrict__ out) {
-  const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (t >= (uint64_t)C * N) return;
-  const uint32_t c = (uint32_t)(t / N), n = (uint32_t)(t % N);
-  AuxWords w = aux_words(seed, kAuxRandom, n, config_id0 + c);
-  float *o = out + t * S;
-  for (uint32_t s = 0; s < S; ++s) o[s] = (float)(aux_next(w) >> 8) * 0x1p-24f;
+// Sec. 4.5: every score replaced by Uniform(0, 1).  Score (c, n, s) is
+// (x >> 8) 2^-24 with x word s of aux stream (RANDOM, canary n) of config id
+// config_id0 + c, i.e. word s % 4 of the Philox block with counter
+// (s / 4, RANDOM << 24 | n, 4 (config_id0 + c) + 3, 0).  A thread makes one
+// such block: four consecutive scores of one row, one 16-byte store when the
+// row's four scores are 16-byte aligned, so a warp writes 512 contiguous
+// bytes.  Grid-stride over the C N ceil(S / 4) blocks.  Below 2^32 blocks
+// the index splits take 32-bit division by multiplication with a
+// precomputed reciprocal: for 32-bit n and d >= 2, n / d is the high 64 bits
+// of n ceil(2^64 / d) (Lemire, Kaser and Kurz, "Faster remainder by direct
+// computation", 2019).  The round keys come precomputed, as in the generator.
+__device__ __forceinline__ uint32_t div_by_recip(uint32_t n, uint64_t recip, uint32_t d) {
+  return d == 1 ? n : (uint32_t)__umul64hi(recip, (uint64_t)n);
+}
+
+constexpr int kRandomBlocksPerSm = 16;
+
+template <bool kIdx32>
+__global__ void __launch_bounds__(256)
+random_scores_kernel(PhiloxRoundKeys rk, uint32_t config_id0, uint32_t N, uint32_t S,
+                     uint64_t total, uint64_t recip_row, uint64_t recip_n,
+                     float *__restrict__ out) {
+  const uint32_t per_row = (S + 3u) / 4u;
+  for (uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+       t += (uint64_t)gridDim.x * blockDim.x) {
+    uint64_t row;
+    uint32_t q, c, n;
+    if (kIdx32) {
+      const uint32_t t32 = (uint32_t)t;
+      const uint32_t r32 = div_by_recip(t32, recip_row, per_row);
+      q = t32 - r32 * per_row;
+      c = div_by_recip(r32, recip_n, N);
+      n = r32 - c * N;
+      row = r32;
+    } else {
+      row = t / per_row;
+      q = (uint32_t)(t - row * per_row);
+      c = (uint32_t)(row / N);
+      n = (uint32_t)(row - (uint64_t)c * N);
+    }
+    const uint4 w = philox4x32_10_rk(
+        make_uint4(q, (kAuxRandom << 24) | (n & 0x00FFFFFFu), 4u * (config_id0 + c) + kStreamAux, 0u),
+        rk);
+    const float v0 = (float)(w.x >> 8) * 0x1p-24f, v1 = (float)(w.y >> 8) * 0x1p-24f;
+    const float v2 = (float)(w.z >> 8) * 0x1p-24f, v3 = (float)(w.w >> 8) * 0x1p-24f;
+    float *o = out + row * S + 4ull * q;
+    if ((S & 3u) == 0 && ((uintptr_t)o & 15u) == 0) {
+      *reinterpret_cast<float4 *>(o) = make_float4(v0, v1, v2, v3);
+    } else {
+      const uint32_t m = min(4u, S - 4u * q);
+      o[0] = v0;
+      if (m > 1) o[1] = v1;
+      if (m > 2) o[2] = v2;
+      if (m > 3) o[3] = v3;
+    }
+  }
 }
 
 // ----------------------------------------------------------------- test views
@@ -687,9 +732,29 @@ cudaError_t launch_generate_propagating(const GenParams &p, float gain, uint16_t
 
 cudaError_t launch_random_scores(uint64_t seed, uint32_t config_id0, uint32_t C, uint32_t N,
                                  uint32_t S, float *out, cudaStream_t stream) {
-  const uint64_t n = (uint64_t)C * N;
-  random_scores_kernel<<<(unsigned)((n + 127) / 128), 128, 0, stream>>>(seed, config_id0, C, N, S,
-                                                                        out);
+  const uint32_t per_row = (S + 3u) / 4u;
+  const uint64_t total = (uint64_t)C * N * per_row;
+  PhiloxRoundKeys rk;
+  uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  for (int r = 0; r < 10; ++r) {
+    rk.k[2 * r] = k0;
+    rk.k[2 * r + 1] = k1;
+    k0 += kPhiloxW0;
+    k1 += kPhiloxW1;
+  }
+  // ceil(2^64 / d) for d >= 2 (unused for d = 1)
+  auto recip = [](uint32_t d) -> uint64_t { return d < 2 ? 0 : UINT64_MAX / d + 1; };
+  DeviceInfo info;
+  if (!device_info(&info)) return cudaGetLastError();
+  const uint64_t blocks = (total + 255) / 256;
+  const uint64_t cap = (uint64_t)info.sm_count * kRandomBlocksPerSm;   // grid-stride beyond
+  const unsigned grid = (unsigned)(blocks < cap ? blocks : cap);
+  if (total < (1ull << 32)) {
+    random_scores_kernel<true><<<grid, 256, 0, stream>>>(rk, config_id0, N, S, total,
+                                                        recip(per_row), recip(N), out);
+  } else {
+    random_scores_kernel<false><<<grid, 256, 0, stream>>>(rk, config_id0, N, S, total, 0, 0, out);
+  }
   return cudaGetLastError();
 }
 

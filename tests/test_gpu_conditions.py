@@ -25,10 +25,24 @@ def cg():
     return m
 
 
-@pytest.mark.parametrize("C,N,S,cid0", [(1, 1, 1, 0), (3, 7, 5, 9), (324, 64, 16, 0), (2, 100, 33, 1000)])
+@pytest.mark.parametrize("C,N,S,cid0", [(1, 1, 1, 0), (3, 7, 5, 9), (324, 64, 16, 0), (2, 100, 33, 1000),
+                                        (5, 3, 4, 7), (2, 9, 12, 3), (1, 1, 6, 0)])
 def test_random_scores_bit_exact(cg, orc, C, N, S, cid0):
     g = cg.cg_random_scores(123, C, N, S, config_id0=cid0).cpu().numpy()
     assert np.array_equal(g, orc.random_scores(123, C, N, S, config_id0=cid0))
+
+
+@pytest.mark.parametrize("C,N,S", [(3, 7, 16), (2, 5, 4), (4, 3, 10)])
+def test_random_scores_unaligned_output(cg, orc, C, N, S):
+    """An output only 4-byte aligned (rows of four scores off the 16-byte
+    grid) takes scalar stores and gives the same bits."""
+    import torch
+    buf = torch.full((C * N * S + 2,), -1.0, dtype=torch.float32, device="cuda")
+    out = buf[1:1 + C * N * S].view(C, N, S)
+    cg.cg_random_scores(5, C, N, S, config_id0=2, out=out)
+    b = buf.cpu().numpy()
+    assert b[0] == -1.0 and b[-1] == -1.0
+    assert np.array_equal(b[1:-1].reshape(C, N, S), orc.random_scores(5, C, N, S, config_id0=2))
 
 
 def test_random_baseline_auroc_matches_oracle(cg, orc):
