@@ -217,10 +217,10 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * seg_len >= 1 (ragged tails handled).  Scores are written to
  * d_scores[stat * stat_stride + n * S + s] (stat_stride >= N * S; pass
  * N * S for a dense [3][N][S] block).  Each element of d_acts and d_refs is
- * read once from HBM.  Sums are accumulated in fp32 per chunk of 16384
- * elements and combined in fp64, so the scores hold their tolerance (rel_l2
- * within 1e-5 relative) for finite element magnitudes between about 1e-18
- * and 1e17: above, the squared sums overflow; below about 1e-19 the squares
+ * read once from HBM.  Sums are accumulated in fp32 per work item of at
+ * most 16384 elements and combined in fp64, so the scores hold their
+ * tolerance (rel_l2 within 1e-5 relative) for finite element magnitudes
+ * between about 1e-18 and 1e17: above, the squared sums overflow; below about 1e-19 the squares
  * fall into fp32's subnormal range and lose precision, and below about
  * 4e-23 they underflow to zero.  A segment whose every squared difference
  * underflows while some difference is nonzero (all |h - a| < 2^-74.5) gets
