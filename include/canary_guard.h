@@ -222,9 +222,10 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * tolerance (rel_l2 within 1e-5 relative) for finite element magnitudes
  * between about 1e-18 and 1e17: above, the squared sums overflow; below
  * about 1e-19 the squares fall into fp32's subnormal range and lose
- * precision, and below about 4e-23 they underflow to zero.  A segment whose every squared difference
- * underflows while some difference is nonzero (all |h - a| < 2^-74.5) gets
- * rel_l2 and cos_dev NaN, never a wrong finite value.  A NaN element
+ * precision, and below about 4e-23 they underflow to zero.  A segment
+ * whose every squared difference underflows while some difference is
+ * nonzero (all |h - a| < 2^-74.5) gets rel_l2 and cos_dev NaN, never a
+ * wrong finite value.  A NaN element
  * makes rel_l2 and cos_dev NaN (max_abs skips it); an infinite live
  * element (fp16 +-inf, which an untrusted hop may send) makes rel_l2 and
  * max_abs +inf and cos_dev NaN.  d_ws: >= cg_drift_workspace_size bytes,
