@@ -227,8 +227,8 @@ cg_status cg_drift_workspace_size(uint32_t n_shards, uint32_t n_canaries,
  * nonzero (all |h - a| < 2^-74.5) gets rel_l2 and cos_dev NaN, never a
  * wrong finite value.  A NaN element makes rel_l2 and cos_dev NaN
  * (max_abs skips it); an infinite live element (fp16 +-inf, which an
- * untrusted hop may send) makes rel_l2 and max_abs +inf and cos_dev NaN.  d_ws: >= cg_drift_workspace_size bytes,
- * 16-byte aligned, scratch.
+ * untrusted hop may send) makes rel_l2 and max_abs +inf and cos_dev NaN.
+ * d_ws: >= cg_drift_workspace_size bytes, 16-byte aligned, scratch.
  */
 cg_status cg_drift_scores(const uint16_t *d_acts, const float *d_refs,
                           uint32_t n_shards, uint32_t n_canaries,
