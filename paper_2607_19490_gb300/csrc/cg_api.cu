@@ -27,6 +27,7 @@ namespace cg {
 
 int drift_occupancy();
 int gen_occupancy();
+int gen_live_occupancy();
 
 bool device_info(DeviceInfo *out) {
   static std::mutex mu;
@@ -44,7 +45,9 @@ bool device_info(DeviceInfo *out) {
     return false;
   info.drift_blocks_per_sm = drift_occupancy();
   info.gen_blocks_per_sm = gen_occupancy();
-  if (info.drift_blocks_per_sm < 1 || info.gen_blocks_per_sm < 1) return false;
+  info.gen_live_blocks_per_sm = gen_live_occupancy();
+  if (info.drift_blocks_per_sm < 1 || info.gen_blocks_per_sm < 1 || info.gen_live_blocks_per_sm < 1)
+    return false;
   if (dev < 64) cache[dev] = info;
   *out = info;
   return true;

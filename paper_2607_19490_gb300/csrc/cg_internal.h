@@ -16,6 +16,7 @@ struct DeviceInfo {
   int sm_count = 0;
   int drift_blocks_per_sm = 0;
   int gen_blocks_per_sm = 0;
+  int gen_live_blocks_per_sm = 0;
 };
 // Cached per current device; returns false on a CUDA error.
 bool device_info(DeviceInfo *out);
