@@ -785,7 +785,8 @@ cudaError_t launch_box_muller_pairs(const uint32_t *words, uint64_t n_pairs, flo
 // memory) still fits beside them.  A caller that scores one configuration
 // while it generates the next on another stream then overlaps the two: the
 // generator is bound by integer/FP32 issue, the drift reduction by HBM.  At
-// 4 blocks per SM instead of 3 the generator alone is about 3 % faster.
+// 4 blocks per SM instead of 3 pass 1 is about 1 % faster alone and the
+// studies 0.2-1.4 % faster, too little to give up that room.
 int gen_occupancy() {
   int n = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gen_refs_kernel<true>, kGenThreads, 0) !=
